@@ -1,0 +1,228 @@
+/*
+ * gf.h - C ABI of the GB300 surrogate forecaster.
+ *
+ * The surrogate of Sec. 2.1 reads x_i = (r, k_i, h) (reference kernel,
+ * candidate kernel, hardware) as one token sequence, generates a brief chain
+ * of reasoning by greedy decoding, and emits a distribution p_i over verdict
+ * tokens.  Its confidence is q_i = max_b p_{i,b}, its predicted verdict is
+ * y_hat_i = argmax_b p_{i,b}, and a forecast is used only when q_i clears a
+ * threshold tau; the remaining candidates are deferred to real GPU
+ * measurement (Sec. 2.1, "Selective Use").
+ *
+ * The language model is a pre-norm decoder-only transformer with RMSNorm,
+ * rotary position embedding (rotate-half, pairs (i, i+hd/2), positions from
+ * 0), grouped-query attention, SwiGLU feed-forward blocks, a final RMSNorm and
+ * an untied LM head; no biases.  Weights are bf16; the residual stream is
+ * fp32; matmuls accumulate in fp32.
+ *
+ * Conventions for every call:
+ *   - Return value: GF_OK (0) or one of the GF_E* codes below; on error the
+ *     outputs are unspecified and gf_last_error() (thread-local) says why.
+ *   - "device" pointers are CUDA global memory of the device the model was
+ *     created on; "host" pointers are ordinary host memory.  The caller owns
+ *     every buffer it passes; no call frees or keeps caller memory beyond
+ *     the call except where stated (gf_create borrows nothing: it copies).
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Device work is enqueued on it asynchronously unless the call
+ *     says it synchronises.
+ *   - Token ids must lie in [0, vocab); lengths must be >= 1.
+ *   - Not thread-safe per model: one host thread drives a model at a time.
+ */
+#ifndef GF_H_
+#define GF_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+  GF_OK = 0,
+  GF_EINVAL = 1,     /* bad argument: shape, id >= vocab, K outside 1..8, tau outside [0,1], bad handle */
+  GF_ECAPACITY = 2,  /* KV page pool, sequence slots or prefill token budget exhausted */
+  GF_ENOMEM = 3,     /* a device or host allocation failed */
+  GF_ECUDA = 4,      /* a CUDA runtime or driver call failed (message in gf_last_error) */
+  GF_ENOTIMPL = 5,   /* configuration the kernels do not support (e.g. head_dim not 64/128) */
+  GF_ETIMEOUT = 6    /* a device-side bounded wait gave up; the kernel returned early */
+};
+
+/* Model shape and resource limits. */
+typedef struct gf_config {
+  int32_t layers;
+  int32_t d_model;     /* multiple of 64 */
+  int32_t n_q;         /* query heads */
+  int32_t n_kv;        /* key/value heads; n_q % n_kv == 0, n_q / n_kv <= 16 */
+  int32_t head_dim;    /* 64 or 128 */
+  int32_t ffn;         /* SwiGLU width */
+  int32_t vocab;
+  float rope_theta;
+  float rms_eps;
+  int32_t max_batch;   /* sequence slots (concurrent sequences), <= 1024 */
+  int32_t max_seq;     /* tokens per sequence, prompt + generated */
+  int64_t max_prefill_tokens; /* largest total prompt tokens of one gf_prefill call */
+  int64_t kv_pages;    /* 64-token pages in the KV pool; 0 = max_batch * ceil(max_seq / 64) */
+} gf_config;
+
+/* Canonical weights, bf16 row-major, rows = output features (as in y = x W^T).
+ * All pointers are device pointers; the per-layer members are HOST arrays of
+ * `layers` device pointers.  Shapes:
+ *   embed [vocab, d]; lm_head [vocab, d]; final_norm [d];
+ *   attn_norm[l], ffn_norm[l] [d];
+ *   wq[l] [n_q*hd, d]; wk[l], wv[l] [n_kv*hd, d]; wo[l] [d, n_q*hd];
+ *   w_gate[l], w_up[l] [ffn, d]; w_down[l] [d, ffn].
+ * gf_create copies them into its own packed layout; the caller may free
+ * them once gf_create returns and its stream has drained. */
+typedef struct gf_weights {
+  const void* embed;
+  const void* lm_head;
+  const void* final_norm;
+  const void* const* attn_norm;
+  const void* const* wq;
+  const void* const* wk;
+  const void* const* wv;
+  const void* const* wo;
+  const void* const* ffn_norm;
+  const void* const* w_gate;
+  const void* const* w_up;
+  const void* const* w_down;
+} gf_weights;
+
+typedef struct gf_model gf_model;
+
+/* Create a model on the current CUDA device: allocates the packed weight
+ * arena, the paged KV pool (page size 64 tokens) and activation buffers for
+ * `max_prefill_tokens`, then packs `w` on `stream` and synchronises it. */
+int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model** out);
+
+/* Free everything the model owns.  Synchronises the device first. */
+void gf_destroy(gf_model* m);
+
+/* Prefill B prompts (Sec. 2.1: the prompt holds reference and candidate
+ * kernel sources and the hardware table as tokens).
+ *   ids          device int32[offsets[B]], prompts packed back to back
+ *   offsets      host int32[B+1], offsets[0] = 0, strictly increasing
+ *   seq_handles  host int32[B] (out): one slot per prompt, for decode/release
+ *   last_logits  device float[B*vocab] or NULL: logits of each prompt's last
+ *                position (those that pick the first generated token)
+ *   next_ids     device int32[B] or NULL: greedy arg max of last_logits
+ *                (lowest id on ties)
+ * Fails with GF_ECAPACITY (nothing allocated) if slots, pages or
+ * max_prefill_tokens are exceeded. */
+int gf_prefill(gf_model* m, int32_t B, const int32_t* ids, const int32_t* offsets, int32_t* seq_handles,
+               float* last_logits, int32_t* next_ids, void* stream);
+
+/* One greedy decode step: feed ids[b] to sequence seq_handles[b] at its next
+ * position, using and extending its paged KV cache.
+ *   seq_handles  host int32[B], distinct live handles
+ *   ids          device int32[B]
+ *   logits       device float[B*vocab] or NULL
+ *   next_ids     device int32[B] or NULL: arg max of the new logits
+ * ids and next_ids may alias (in-place greedy loop).  GF_ECAPACITY if a
+ * sequence would exceed max_seq or the pool has no free page. */
+int gf_decode_step(gf_model* m, int32_t B, const int32_t* seq_handles, const int32_t* ids, float* logits,
+                   int32_t* next_ids, void* stream);
+
+/* Return the slots and KV pages of the given sequences to the pool.  Work
+ * already enqueued that reads them must be ordered before any later call
+ * that reuses them (all calls of one model on one stream are). */
+int gf_release(gf_model* m, int32_t B, const int32_t* seq_handles);
+
+/* The whole forecast of Sec. 2.1 for a batch of candidates:
+ *   prompt_i = incumbent ids ‖ candidate ids  (x_i = (r, k_i, h));
+ *   prefill, then n_decode greedy steps (the reasoning trace), then on the
+ *   logits of the last step (the last prompt position if n_decode == 0):
+ *     p[i,:] = softmax(logits[i, verdict_ids[0..K-1]])   (restricted softmax)
+ *     conf[i] = max_b p[i,b]                              (q_i)
+ *     verdict_arg[i] = argmax_b p[i,b], lowest b on ties  (y_hat_i)
+ *     defer[i] = conf[i] < tau                            (measure on the GPU)
+ *   Slots are released before returning.
+ *   inc_ids, cand_ids          device int32, packed
+ *   inc_offsets, cand_offsets  host int32[B+1]; each item's total length >= 1
+ *   verdict_ids                host int32[K], 1 <= K <= 8, ids < vocab
+ *   p [B*K], conf [B] float; verdict_arg [B] int32; defer [B] uint8: device
+ *   tokens  device int32[B*n_decode] or NULL: the generated tokens, row-major
+ *   final_logits device float[B*vocab] or NULL: the logits the verdict reads */
+int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                      const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                      const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                      int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, float* final_logits, void* stream);
+
+/* gf_forecast_batch with every array in host memory: copies the ids to the
+ * device, runs the forecast, copies p/conf/verdict_arg/defer (and tokens if
+ * non-NULL) back, and synchronises `stream` before returning. */
+int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                           const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                           const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                           int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, void* stream);
+
+/* Stand-alone verdict step (Sec. 2.1) on caller logits:
+ *   logits device float[B*ld] (row stride ld >= max verdict id + 1);
+ *   verdict_ids host int32[K]; outputs as in gf_forecast_batch. */
+int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdict_ids, int32_t K, float tau,
+               float* p, float* conf, int32_t* verdict_arg, uint8_t* defer, void* stream);
+
+/* ---- building blocks --------------------------------------------------------
+ * The dense contraction every projection of the forward pass uses, exposed on
+ * its own: out[M,N] (op)= A[M,K] . W[N,K]^T on the tcgen05 tensor cores.
+ *   A, W   device bf16, row-major (K contiguous); K % 64 == 0, N % 32 == 0
+ *   mode   GF_GEMM_STORE_F32:  out (float, row stride ldo) = acc
+ *          GF_GEMM_ADD_F32:    out += acc (non-atomic, as on the residual stream)
+ *          GF_GEMM_ATOMIC_F32: out += acc with atomics (split-K partial sums)
+ *          GF_GEMM_STORE_BF16: out (bf16) = acc
+ *          GF_GEMM_SWIGLU:     W rows hold blocks of 64 gate rows followed by 64
+ *                              up rows; out (bf16, N/2 columns) = silu(gate) * up
+ *   bn     tile width 64, 128 or 256, or 0 to choose; splits: split-K factor
+ *          (only with GF_GEMM_ATOMIC_F32), 0 to choose.
+ * Enqueued on `stream`; a device-side timeout is reported by gf_gemm_status. */
+enum { GF_GEMM_STORE_F32 = 0, GF_GEMM_ADD_F32 = 1, GF_GEMM_ATOMIC_F32 = 2, GF_GEMM_STORE_BF16 = 3,
+       GF_GEMM_SWIGLU = 4 };
+int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
+                 int32_t mode, int32_t bn, int32_t splits, void* stream);
+/* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16 launch gave up waiting. */
+int gf_gemm_status(void* stream);
+
+/* ---- measurement ------------------------------------------------------------
+ * Kernel classes whose launches can be bracketed by CUDA events (on the
+ * launching stream) for live timing inside a run. */
+enum { GF_PROF_PREFILL_GEMM = 0, GF_PROF_DECODE_GEMM = 1, GF_PROF_PREFILL_ATTN = 2, GF_PROF_DECODE_ATTN = 3,
+       GF_PROF_KINDS = 4 };
+/* Time every launch of the classes whose bit is set in `mask` (0 = off). */
+int gf_profile_enable(gf_model* m, uint32_t mask);
+/* Synchronise the device and return, for class `kind` since the last read:
+ * launches, summed kernel milliseconds, algorithmic FLOPs (2*M*N*K for a
+ * GEMM, 4*hd per visible query-key pair for attention) and algorithmic HBM
+ * bytes (operands read once, outputs written once); then reset the class. */
+int gf_profile_read(gf_model* m, int32_t kind, int64_t* launches, double* ms, double* flops, double* bytes);
+
+/* ---- inspection hooks (parity tests at full size) -------------------------
+ * gf_debug_capture arms a copy, during the NEXT gf_prefill or gf_decode_step,
+ * of the fp32 residual stream entering layer `layer` (layer == layers: the
+ * final hidden state before the final RMSNorm) for batch item `item`:
+ * prefill copies that prompt's rows [len, d], decode its single row [1, d],
+ * into device float dst (capacity `cap_rows` rows).  Up to 8 captures may be
+ * armed at once; each fires once.  GF_EINVAL on bad layer/item/cap. */
+int gf_debug_capture(gf_model* m, int32_t layer, int32_t item, float* dst, int64_t cap_rows);
+
+/* Copy the cached keys and values of sequence `handle` at positions
+ * [start, start+n) of layer `layer` into dense device bf16 arrays
+ * k_dst, v_dst [n, n_kv, head_dim].  Enqueued on `stream`. */
+int gf_debug_read_kv(gf_model* m, int32_t layer, int32_t handle, int32_t start, int32_t n, void* k_dst,
+                     void* v_dst, void* stream);
+
+/* Synchronise `stream` and report a device-side timeout recorded by any
+ * kernel of this model since the last call (GF_ETIMEOUT), then clear it. */
+int gf_device_status(gf_model* m, void* stream);
+
+/* Number of kernels this model has launched since creation (for accounting). */
+int64_t gf_launch_count(const gf_model* m);
+
+/* Thread-local description of the last error; never NULL. */
+const char* gf_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GF_H_ */

@@ -1,0 +1,342 @@
+"""GB300 surrogate forecaster: thin Python binding of the C ABI in include/gf.h.
+
+Every step of the forward pass, the greedy decode and the verdict/defer step
+runs in the CUDA library ``_build/libgf.so`` (hand-written sm_103a kernels).
+This module only marshals arguments: functions named like the C entry points
+take raw pointers and sizes; ``Model`` wraps them for torch tensors, which
+serve only as device memory and streams.  There is no fallback path: if the
+library is missing, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libgf.so")
+
+GF_OK, GF_EINVAL, GF_ECAPACITY, GF_ENOMEM, GF_ECUDA, GF_ENOTIMPL, GF_ETIMEOUT = range(7)
+
+_c_i32, _c_i64, _c_f32, _p = ctypes.c_int32, ctypes.c_int64, ctypes.c_float, ctypes.c_void_p
+
+
+class GfError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__(f"gf error {code}: {msg}")
+        self.code = code
+
+
+class gf_config(ctypes.Structure):
+    _fields_ = [("layers", _c_i32), ("d_model", _c_i32), ("n_q", _c_i32), ("n_kv", _c_i32), ("head_dim", _c_i32),
+                ("ffn", _c_i32), ("vocab", _c_i32), ("rope_theta", _c_f32), ("rms_eps", _c_f32),
+                ("max_batch", _c_i32), ("max_seq", _c_i32), ("max_prefill_tokens", _c_i64), ("kv_pages", _c_i64)]
+
+
+_PP = ctypes.POINTER(_p)
+
+
+class gf_weights(ctypes.Structure):
+    _fields_ = [("embed", _p), ("lm_head", _p), ("final_norm", _p), ("attn_norm", _PP), ("wq", _PP), ("wk", _PP),
+                ("wv", _PP), ("wo", _PP), ("ffn_norm", _PP), ("w_gate", _PP), ("w_up", _PP), ("w_down", _PP)]
+
+
+EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_release", "gf_forecast_batch",
+           "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
+           "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
+           "gf_profile_read"]
+
+GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
+GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN = range(4)
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load libgf.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"CUDA library {path} is missing: build it with paper_2605_31464_gb300._build.build()")
+    lib = ctypes.CDLL(path)
+    sig = {
+        "gf_create": ([ctypes.POINTER(gf_config), ctypes.POINTER(gf_weights), _p, ctypes.POINTER(_p)], ctypes.c_int),
+        "gf_destroy": ([_p], None),
+        "gf_prefill": ([_p, _c_i32, _p, _p, _p, _p, _p, _p], ctypes.c_int),
+        "gf_decode_step": ([_p, _c_i32, _p, _p, _p, _p, _p], ctypes.c_int),
+        "gf_release": ([_p, _c_i32, _p], ctypes.c_int),
+        "gf_forecast_batch": ([_p, _c_i32, _p, _p, _p, _p, _c_i32, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p, _p, _p],
+                              ctypes.c_int),
+        "gf_forecast_batch_host": ([_p, _c_i32, _p, _p, _p, _p, _c_i32, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p, _p],
+                                   ctypes.c_int),
+        "gf_verdict": ([_c_i32, _p, _c_i64, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
+        "gf_debug_capture": ([_p, _c_i32, _c_i32, _p, _c_i64], ctypes.c_int),
+        "gf_debug_read_kv": ([_p, _c_i32, _c_i32, _c_i32, _c_i32, _p, _p, _p], ctypes.c_int),
+        "gf_device_status": ([_p, _p], ctypes.c_int),
+        "gf_launch_count": ([_p], _c_i64),
+        "gf_last_error": ([], ctypes.c_char_p),
+        "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _p], ctypes.c_int),
+        "gf_gemm_status": ([_p], ctypes.c_int),
+        "gf_profile_enable": ([_p, ctypes.c_uint32], ctypes.c_int),
+        "gf_profile_read": ([_p, _c_i32, ctypes.POINTER(_c_i64), ctypes.POINTER(ctypes.c_double),
+                             ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
+    }
+    for name, (args, res) in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = res
+    _lib = lib
+    return lib
+
+
+def _check(rc: int):
+    if rc != GF_OK:
+        raise GfError(rc, load().gf_last_error().decode())
+
+
+# ---------------------------------------------------------------- raw entry points (pointers and sizes)
+
+def gf_create(cfg: gf_config, weights: gf_weights, stream: int) -> int:
+    out = _p()
+    _check(load().gf_create(ctypes.byref(cfg), ctypes.byref(weights), stream, ctypes.byref(out)))
+    return out.value
+
+
+def gf_destroy(model: int) -> None:
+    load().gf_destroy(model)
+
+
+def gf_prefill(model, B, ids, offsets, seq_handles, last_logits, next_ids, stream):
+    _check(load().gf_prefill(model, B, ids, offsets, seq_handles, last_logits, next_ids, stream))
+
+
+def gf_decode_step(model, B, seq_handles, ids, logits, next_ids, stream):
+    _check(load().gf_decode_step(model, B, seq_handles, ids, logits, next_ids, stream))
+
+
+def gf_release(model, B, seq_handles):
+    _check(load().gf_release(model, B, seq_handles))
+
+
+def gf_forecast_batch(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, K, tau, p,
+                      conf, verdict_arg, defer, tokens, final_logits, stream):
+    _check(load().gf_forecast_batch(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids,
+                                    K, tau, p, conf, verdict_arg, defer, tokens, final_logits, stream))
+
+
+def gf_forecast_batch_host(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, K, tau, p,
+                           conf, verdict_arg, defer, tokens, stream):
+    _check(load().gf_forecast_batch_host(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode,
+                                         verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens, stream))
+
+
+def gf_verdict(B, logits, ld, verdict_ids, K, tau, p, conf, verdict_arg, defer, stream):
+    _check(load().gf_verdict(B, logits, ld, verdict_ids, K, tau, p, conf, verdict_arg, defer, stream))
+
+
+def gf_debug_capture(model, layer, item, dst, cap_rows):
+    _check(load().gf_debug_capture(model, layer, item, dst, cap_rows))
+
+
+def gf_debug_read_kv(model, layer, handle, start, n, k_dst, v_dst, stream):
+    _check(load().gf_debug_read_kv(model, layer, handle, start, n, k_dst, v_dst, stream))
+
+
+def gf_device_status(model, stream):
+    _check(load().gf_device_status(model, stream))
+
+
+def gf_launch_count(model) -> int:
+    return int(load().gf_launch_count(model))
+
+
+def gf_last_error() -> str:
+    return load().gf_last_error().decode()
+
+
+def gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, stream):
+    _check(load().gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, stream))
+
+
+def gf_gemm_status(stream):
+    _check(load().gf_gemm_status(stream))
+
+
+def gf_profile_enable(model, mask):
+    _check(load().gf_profile_enable(model, mask))
+
+
+def gf_profile_read(model, kind):
+    n, ms, fl, by = _c_i64(), ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+    _check(load().gf_profile_read(model, kind, ctypes.byref(n), ctypes.byref(ms), ctypes.byref(fl), ctypes.byref(by)))
+    return dict(launches=n.value, ms=ms.value, flops=fl.value, bytes=by.value)
+
+
+def gemm(A, W, out, mode=GF_GEMM_STORE_F32, bn=0, splits=0, stream=None):
+    """out (op)= A . W^T on the tensor cores (A [M,K], W [N,K] bf16 CUDA tensors)."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    M, K = A.shape
+    N = W.shape[0]
+    gf_gemm_bf16(A.data_ptr(), W.data_ptr(), M, N, K, out.data_ptr(), out.stride(0), mode, bn, splits, s.cuda_stream)
+
+
+# ---------------------------------------------------------------- torch-facing wrapper
+
+def _i32_host(a) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(a, dtype=np.int32))
+
+
+def _ptr(a: np.ndarray):
+    return a.ctypes.data_as(_p)
+
+
+class Model:
+    """A model on the current CUDA device.
+
+    ``shape`` has the fields of gf_config's model part (layers, d_model, n_q,
+    n_kv, head_dim, ffn, vocab, rope_theta, rms_eps).  ``weights`` maps
+    names to bf16 CUDA tensors: embed, lm_head, final_norm and per layer
+    lists attn_norm, wq, wk, wv, wo, ffn_norm, w_gate, w_up, w_down.
+    """
+
+    def __init__(self, shape, weights: dict, max_batch: int, max_seq: int, max_prefill_tokens: int,
+                 kv_pages: int = 0, stream=None):
+        import torch
+        self.torch = torch
+        self.shape = shape
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        cfg = gf_config(layers=shape.layers, d_model=shape.d_model, n_q=shape.n_q, n_kv=shape.n_kv,
+                        head_dim=shape.head_dim, ffn=shape.ffn, vocab=shape.vocab, rope_theta=shape.rope_theta,
+                        rms_eps=shape.rms_eps, max_batch=max_batch, max_seq=max_seq,
+                        max_prefill_tokens=max_prefill_tokens, kv_pages=kv_pages)
+        L = shape.layers
+
+        def arr(name):
+            a = (_p * L)(*[t.data_ptr() for t in weights[name]])
+            return ctypes.cast(a, _PP), a
+
+        keep = {}
+        fields = {}
+        for name in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down"):
+            fields[name], keep[name] = arr(name)
+        w = gf_weights(embed=weights["embed"].data_ptr(), lm_head=weights["lm_head"].data_ptr(),
+                       final_norm=weights["final_norm"].data_ptr(), **fields)
+        self.cfg = cfg
+        self.max_batch, self.max_seq = max_batch, max_seq
+        self.handle = gf_create(cfg, w, self.stream.cuda_stream)
+
+    @property
+    def s(self) -> int:
+        return self.stream.cuda_stream
+
+    def close(self):
+        if getattr(self, "handle", None):
+            gf_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # -- calls
+    def prefill(self, ids, offsets, want_logits: bool = True):
+        torch = self.torch
+        off = _i32_host(offsets)
+        B = len(off) - 1
+        handles = np.zeros(B, dtype=np.int32)
+        logits = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
+        nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+        gf_prefill(self.handle, B, ids.data_ptr(), _ptr(off), _ptr(handles),
+                   logits.data_ptr() if logits is not None else None, nxt.data_ptr(), self.s)
+        return handles, logits, nxt
+
+    def decode_step(self, handles, ids, want_logits: bool = True):
+        torch = self.torch
+        h = _i32_host(handles)
+        B = len(h)
+        logits = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
+        nxt = torch.empty(B, dtype=torch.int32, device="cuda")
+        gf_decode_step(self.handle, B, _ptr(h), ids.data_ptr(), logits.data_ptr() if logits is not None else None,
+                       nxt.data_ptr(), self.s)
+        return logits, nxt
+
+    def release(self, handles):
+        h = _i32_host(handles)
+        gf_release(self.handle, len(h), _ptr(h))
+
+    def forecast_batch(self, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, tau,
+                       want_tokens=True, want_logits=False):
+        torch = self.torch
+        io, co, vid = _i32_host(inc_offsets), _i32_host(cand_offsets), _i32_host(verdict_ids)
+        B, K = len(io) - 1, len(vid)
+        p = torch.empty(B, K, dtype=torch.float32, device="cuda")
+        conf = torch.empty(B, dtype=torch.float32, device="cuda")
+        arg = torch.empty(B, dtype=torch.int32, device="cuda")
+        defer = torch.empty(B, dtype=torch.uint8, device="cuda")
+        toks = torch.empty(B, max(n_decode, 1), dtype=torch.int32, device="cuda") if want_tokens else None
+        lg = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
+        gf_forecast_batch(self.handle, B, inc_ids.data_ptr(), _ptr(io), cand_ids.data_ptr(), _ptr(co), n_decode,
+                          _ptr(vid), K, float(tau), p.data_ptr(), conf.data_ptr(), arg.data_ptr(), defer.data_ptr(),
+                          toks.data_ptr() if toks is not None and n_decode > 0 else None,
+                          lg.data_ptr() if lg is not None else None, self.s)
+        return dict(p=p, conf=conf, arg=arg, defer=defer, tokens=toks, logits=lg)
+
+    def forecast_batch_host(self, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, tau,
+                            want_tokens=True):
+        inc, cand = _i32_host(inc_ids), _i32_host(cand_ids)
+        io, co, vid = _i32_host(inc_offsets), _i32_host(cand_offsets), _i32_host(verdict_ids)
+        B, K = len(io) - 1, len(vid)
+        p = np.zeros((B, K), dtype=np.float32)
+        conf = np.zeros(B, dtype=np.float32)
+        arg = np.zeros(B, dtype=np.int32)
+        defer = np.zeros(B, dtype=np.uint8)
+        toks = np.zeros((B, max(n_decode, 1)), dtype=np.int32) if want_tokens else None
+        gf_forecast_batch_host(self.handle, B, _ptr(inc), _ptr(io), _ptr(cand), _ptr(co), n_decode, _ptr(vid), K,
+                               float(tau), _ptr(p), _ptr(conf), _ptr(arg), _ptr(defer),
+                               _ptr(toks) if toks is not None and n_decode > 0 else None, self.s)
+        return dict(p=p, conf=conf, arg=arg, defer=defer, tokens=toks)
+
+    def capture(self, layer: int, item: int, rows: int):
+        """Arm a copy of the residual stream entering `layer` for batch item `item` (next call)."""
+        buf = self.torch.zeros(rows, self.shape.d_model, dtype=self.torch.float32, device="cuda")
+        gf_debug_capture(self.handle, layer, item, buf.data_ptr(), rows)
+        return buf
+
+    def read_kv(self, layer: int, handle: int, start: int, n: int):
+        torch = self.torch
+        k = torch.empty(n, self.shape.n_kv, self.shape.head_dim, dtype=torch.bfloat16, device="cuda")
+        v = torch.empty_like(k)
+        gf_debug_read_kv(self.handle, layer, handle, start, n, k.data_ptr(), v.data_ptr(), self.s)
+        return k, v
+
+    def status(self):
+        gf_device_status(self.handle, self.s)
+
+    def launch_count(self) -> int:
+        return gf_launch_count(self.handle)
+
+    def profile(self, mask: int):
+        gf_profile_enable(self.handle, mask)
+
+    def profile_read(self, kind: int) -> dict:
+        return gf_profile_read(self.handle, kind)
+
+
+def verdict(logits, verdict_ids, tau, stream=None):
+    """Stand-alone verdict step on a [B, V] float32 CUDA tensor."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    vid = _i32_host(verdict_ids)
+    B, K = logits.shape[0], len(vid)
+    p = torch.empty(B, K, dtype=torch.float32, device=logits.device)
+    conf = torch.empty(B, dtype=torch.float32, device=logits.device)
+    arg = torch.empty(B, dtype=torch.int32, device=logits.device)
+    defer = torch.empty(B, dtype=torch.uint8, device=logits.device)
+    gf_verdict(B, logits.data_ptr(), logits.stride(0), _ptr(vid), K, float(tau), p.data_ptr(), conf.data_ptr(),
+               arg.data_ptr(), defer.data_ptr(), s.cuda_stream)
+    return p, conf, arg, defer

@@ -1,0 +1,285 @@
+// Decode attention over the paged KV cache: one new query token per sequence.
+//
+// Grid (split, kv_head, sequence).  A CTA takes `chunk` keys of one sequence
+// and one KV head and serves every query head of that group at once (the G
+// heads of a GQA group are the 16 rows of a warp MMA, zero-padded), so each
+// K/V page is read from HBM once per step.  Pages (64 tokens x head_dim)
+// arrive by TMA, double-buffered; warp w takes keys 16w..16w+15 of each page.
+// Each CTA writes an unnormalised partial (running max, running sum, sum of
+// p.v) for its chunk; attn_combine merges the chunks of a sequence.
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace gf {
+
+template <int HD>
+struct DecodeCfg {
+  static constexpr int HALVES = HD / 64;
+  static constexpr int PAGE_HALF = 64 * 128;        // one 64-column half of a page
+  static constexpr int PAGE_BYTES = 64 * HD * 2;    // one page of K (or V) for one head
+  static constexpr int Q_BYTES = 16 * HD * 2;
+  // smem: Q [HALVES][16][128 B] | K[2] | V[2] | barriers ; the K/V area is reused to combine warps
+  static constexpr int SMEM = 1024 + Q_BYTES + 4 * PAGE_BYTES + 64;
+};
+
+template <int HD>
+__global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant__ CUtensorMap tmK,
+                                                          const __grid_constant__ CUtensorMap tmV,
+                                                          const DecodeAttnArgs a) {
+  using C = DecodeCfg<HD>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + C::Q_BYTES;
+  uint8_t* sV = sK + 2 * C::PAGE_BYTES;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + 2 * C::PAGE_BYTES);  // [2]
+
+  const int split = blockIdx.x;
+  const int kvh = blockIdx.y;
+  const int b = blockIdx.z;
+  const int slot = a.handles[b];
+  const int ctx = a.seq_len[slot] + 1;
+  const int k0 = split * a.chunk;
+  if (k0 >= ctx) return;
+  const int k1 = min(k0 + a.chunk, ctx);
+  const int p0 = k0 >> 6;
+  const int n_pages = ((k1 - 1) >> 6) - p0 + 1;
+  const int G = a.n_q / a.n_kv;
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int32_t* pages = a.block_table + (int64_t)slot * a.max_pages;
+
+  auto issue = [&](int i) {
+    const int buf = i & 1;
+    const int64_t row = a.layer_row0 + ((int64_t)pages[p0 + i] * a.n_kv + kvh) * 64;
+    mbar_arrive_expect_tx(&bar[buf], 2 * C::PAGE_BYTES);
+#pragma unroll
+    for (int h = 0; h < C::HALVES; ++h) {
+      tma_load_2d(sK + buf * C::PAGE_BYTES + h * C::PAGE_HALF, &tmK, &bar[buf], h * 64, (int)row);
+      tma_load_2d(sV + buf * C::PAGE_BYTES + h * C::PAGE_HALF, &tmV, &bar[buf], h * 64, (int)row);
+    }
+  };
+
+  if (threadIdx.x == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    fence_mbar_init();
+    fence_async_smem();
+    issue(0);
+    if (n_pages > 1) issue(1);
+  }
+  // Q rows of this group (zero rows beyond G), 16-byte chunks, swizzled like TMA.
+  for (int c = threadIdx.x; c < 16 * (HD / 8); c += blockDim.x) {
+    const int r = c / (HD / 8), ch = c % (HD / 8);
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (r < G) v = *reinterpret_cast<const uint4*>(a.q + (int64_t)b * a.ldq + (kvh * G + r) * HD + ch * 8);
+    *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (16 * 128) + sw128(r, ch & 7)) = v;
+  }
+  __syncthreads();
+
+  uint32_t qa[HD / 16][4];
+  {
+    const int r = (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const int chunk = kk * 2 + (lane >> 4);
+      ldsm_x4(smem_u32(sQ + (chunk >> 3) * (16 * 128)) + sw128(r, chunk & 7), qa[kk][0], qa[kk][1], qa[kk][2],
+              qa[kk][3]);
+    }
+  }
+
+  float o[HD / 8][4];
+#pragma unroll
+  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
+  float m_run[2] = {-INFINITY, -INFINITY};
+  float l_run[2] = {0.f, 0.f};
+  const int t4 = lane & 3;
+  bool ok = true;
+  int i_fail = 0;
+
+  for (int i = 0; i < n_pages; ++i) {
+    const int buf = i & 1;
+    if (!mbar_wait(&bar[buf], (i >> 1) & 1, a.err)) {
+      ok = false;
+      i_fail = i;
+      break;
+    }
+    const uint8_t* k_t = sK + buf * C::PAGE_BYTES;
+    const uint8_t* v_t = sV + buf * C::PAGE_BYTES;
+    float s[2][4];
+#pragma unroll
+    for (int n = 0; n < 2; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
+#pragma unroll
+    for (int kk = 0; kk < HD / 16; ++kk) {
+      const int key = warp * 16 + (lane & 7) + (lane >> 4) * 8;
+      const int chunk = kk * 2 + ((lane >> 3) & 1);
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4(smem_u32(k_t + (chunk >> 3) * C::PAGE_HALF) + sw128(key, chunk & 7), b0, b1, b2, b3);
+      mma_bf16_16816(s[0], qa[kk], b0, b1);
+      mma_bf16_16816(s[1], qa[kk], b2, b3);
+    }
+    const int key_base = (p0 + i) * 64 + warp * 16;
+    float mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int n = 0; n < 2; ++n) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = key_base + n * 8 + 2 * t4 + (e & 1);
+        float v = s[n][e] * a.scale_log2;
+        if (key < k0 || key >= k1) v = -INFINITY;
+        s[n][e] = v;
+        mx[e >> 1] = fmaxf(mx[e >> 1], v);
+      }
+    }
+    float corr[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
+      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
+      const float m_new = fmaxf(m_run[r], mx[r]);
+      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
+      corr[r] = exp2f(m_run[r] - m_use);
+      m_run[r] = m_new;
+      mx[r] = m_use;
+    }
+    float rs[2] = {0.f, 0.f};
+#pragma unroll
+    for (int n = 0; n < 2; ++n) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const float pv = exp2f(s[n][e] - mx[e >> 1]);
+        s[n][e] = pv;
+        rs[e >> 1] += pv;
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) l_run[r] = l_run[r] * corr[r] + rs[r];
+#pragma unroll
+    for (int d = 0; d < HD / 8; ++d) {
+      o[d][0] *= corr[0];
+      o[d][1] *= corr[0];
+      o[d][2] *= corr[1];
+      o[d][3] *= corr[1];
+    }
+    uint32_t pa[4];
+    pa[0] = pack_bf16(s[0][0], s[0][1]);
+    pa[1] = pack_bf16(s[0][2], s[0][3]);
+    pa[2] = pack_bf16(s[1][0], s[1][1]);
+    pa[3] = pack_bf16(s[1][2], s[1][3]);
+#pragma unroll
+    for (int dp = 0; dp < HD / 16; ++dp) {
+      const int key = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+      const int chunk = dp * 2 + (lane >> 4);
+      uint32_t b0, b1, b2, b3;
+      ldsm_x4_t(smem_u32(v_t + (chunk >> 3) * C::PAGE_HALF) + sw128(key, chunk & 7), b0, b1, b2, b3);
+      mma_bf16_16816(o[2 * dp], pa, b0, b1);
+      mma_bf16_16816(o[2 * dp + 1], pa, b2, b3);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && i + 2 < n_pages) issue(i + 2);
+  }
+
+  if (!ok) {
+    if (threadIdx.x == 0)
+      for (int i = i_fail; i < min(n_pages, i_fail + 2); ++i) mbar_wait_drain(&bar[i & 1], (i >> 1) & 1);
+    return;
+  }
+
+  // ---- combine the four warps (K/V buffers are free now)
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 1);
+    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 2);
+  }
+  float* red_o = reinterpret_cast<float*>(sK);          // [4 warps][16 rows][HD]
+  float* red_ml = red_o + 4 * 16 * HD;                  // [4 warps][16 rows][2]
+  const int g = lane >> 2;
+#pragma unroll
+  for (int d = 0; d < HD / 8; ++d) {
+    const int col = d * 8 + 2 * t4;
+    red_o[(warp * 16 + g) * HD + col] = o[d][0];
+    red_o[(warp * 16 + g) * HD + col + 1] = o[d][1];
+    red_o[(warp * 16 + g + 8) * HD + col] = o[d][2];
+    red_o[(warp * 16 + g + 8) * HD + col + 1] = o[d][3];
+  }
+  if (t4 == 0) {
+    red_ml[(warp * 16 + g) * 2] = m_run[0];
+    red_ml[(warp * 16 + g) * 2 + 1] = l_run[0];
+    red_ml[(warp * 16 + g + 8) * 2] = m_run[1];
+    red_ml[(warp * 16 + g + 8) * 2 + 1] = l_run[1];
+  }
+  __syncthreads();
+  const int64_t part = ((int64_t)b * a.n_kv + kvh) * a.max_splits + split;
+  for (int idx = threadIdx.x; idx < G * HD; idx += blockDim.x) {
+    const int r = idx / HD, d = idx % HD;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) M = fmaxf(M, red_ml[(w * 16 + r) * 2]);
+    float L = 0.f, O = 0.f;
+#pragma unroll
+    for (int w = 0; w < 4; ++w) {
+      const float mw = red_ml[(w * 16 + r) * 2];
+      const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+      L += red_ml[(w * 16 + r) * 2 + 1] * f;
+      O += red_o[(w * 16 + r) * HD + d] * f;
+    }
+    a.part_o[(part * 16 + r) * HD + d] = O;
+    if (d == 0) {
+      a.part_ml[(part * 16 + r) * 2] = M;
+      a.part_ml[(part * 16 + r) * 2 + 1] = L;
+    }
+  }
+}
+
+// Merge the per-chunk partials of each (sequence, query head) and normalise.
+template <int HD>
+__global__ void attn_combine_kernel(const DecodeAttnArgs a) {
+  const int b = blockIdx.x / a.n_q;
+  const int h = blockIdx.x % a.n_q;
+  const int G = a.n_q / a.n_kv;
+  const int kvh = h / G, r = h % G;
+  const int ctx = a.seq_len[a.handles[b]] + 1;
+  const int n_splits = (ctx + a.chunk - 1) / a.chunk;
+  const int64_t base = ((int64_t)b * a.n_kv + kvh) * a.max_splits;
+  float M = -INFINITY;
+  for (int s = 0; s < n_splits; ++s) M = fmaxf(M, a.part_ml[((base + s) * 16 + r) * 2]);
+  for (int d = threadIdx.x; d < HD; d += blockDim.x) {
+    float L = 0.f, O = 0.f;
+    for (int s = 0; s < n_splits; ++s) {
+      const float ms = a.part_ml[((base + s) * 16 + r) * 2];
+      const float f = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
+      L += a.part_ml[((base + s) * 16 + r) * 2 + 1] * f;
+      O += a.part_o[((base + s) * 16 + r) * HD + d] * f;
+    }
+    a.out[(int64_t)b * a.ldo + h * HD + d] = __float2bfloat16(L > 0.f ? O / L : 0.f);
+  }
+}
+
+template <int HD>
+static cudaError_t launch_hd(const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a, int B,
+                             cudaStream_t s) {
+  static bool configured = false;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         DecodeCfg<HD>::SMEM);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  if (B == 0) return cudaSuccess;
+  dim3 grid(a.max_splits, a.n_kv, B);
+  attn_decode_kernel<HD><<<grid, 128, DecodeCfg<HD>::SMEM, s>>>(tmK, tmV, a);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  attn_combine_kernel<HD><<<B * a.n_q, HD, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a,
+                               int B, cudaStream_t s) {
+  if (a.n_q / a.n_kv > 16) return cudaErrorInvalidValue;
+  if (hd == 128) return launch_hd<128>(tmK, tmV, a, B, s);
+  if (hd == 64) return launch_hd<64>(tmK, tmV, a, B, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace gf

@@ -1,0 +1,74 @@
+// Host launchers for the tcgen05 GEMM (one template instantiation per tile
+// width and epilogue).
+#include "gemm_tc.cuh"
+#include "kernels.h"
+
+namespace gf {
+
+int gemm_num_stages(int bn) {
+  return bn == 256 ? GemmCfg<256>::STAGES : (bn == 128 ? GemmCfg<128>::STAGES : GemmCfg<64>::STAGES);
+}
+int gemm_smem_bytes(int bn) {
+  return bn == 256 ? GemmCfg<256>::SMEM_BYTES : (bn == 128 ? GemmCfg<128>::SMEM_BYTES : GemmCfg<64>::SMEM_BYTES);
+}
+
+template <int BN, int MODE>
+static cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int grid,
+                              cudaStream_t s) {
+  static bool configured = false;
+  auto kern = gemm_tc_kernel<BN, MODE>;
+  if (!configured) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    configured = true;
+  }
+  kern<<<grid, GemmCfg<BN>::THREADS, GemmCfg<BN>::SMEM_BYTES, s>>>(tmA, tmB, p);
+  return cudaGetLastError();
+}
+
+template <int BN>
+static cudaError_t dispatch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int mode,
+                                 int grid, cudaStream_t s) {
+  switch (mode) {
+    case kStoreF32: return launch_one<BN, kStoreF32>(tmA, tmB, p, grid, s);
+    case kAddF32: return launch_one<BN, kAddF32>(tmA, tmB, p, grid, s);
+    case kAtomicF32: return launch_one<BN, kAtomicF32>(tmA, tmB, p, grid, s);
+    case kStoreBF16: return launch_one<BN, kStoreBF16>(tmA, tmB, p, grid, s);
+    case kSwiGLU:
+      if (BN >= 128) return launch_one<(BN >= 128 ? BN : 128), kSwiGLU>(tmA, tmB, p, grid, s);
+      return cudaErrorInvalidValue;
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
+                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s) {
+  if (M <= 0 || N <= 0) return cudaSuccess;
+  if (K % 64 != 0 || N % 32 != 0) return cudaErrorInvalidValue;
+  GemmArgs p;
+  p.M = M;
+  p.N = N;
+  p.K = K;
+  p.num_m = (M + 127) / 128;
+  p.num_n = (N + bn - 1) / bn;
+  p.kb_total = K / 64;
+  if (splits < 1) splits = 1;
+  if (splits > p.kb_total) splits = p.kb_total;
+  p.kb_per_split = (p.kb_total + splits - 1) / splits;
+  p.splits = (p.kb_total + p.kb_per_split - 1) / p.kb_per_split;  // no empty split
+  p.group_m = 16;
+  p.out = out;
+  p.ldo = ldo;
+  p.err = err;
+  const int tiles = p.num_m * p.num_n * p.splits;
+  if (grid > tiles) grid = tiles;
+  if (grid < 1) grid = 1;
+  switch (bn) {
+    case 64: return dispatch_mode<64>(tmA, tmB, p, mode, grid, s);
+    case 128: return dispatch_mode<128>(tmA, tmB, p, mode, grid, s);
+    case 256: return dispatch_mode<256>(tmA, tmB, p, mode, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace gf

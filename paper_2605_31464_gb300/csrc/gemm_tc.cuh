@@ -1,0 +1,300 @@
+// bf16 GEMM on the 5th-generation tensor cores:  C[M,N] (op)= A[M,K] . B[N,K]^T
+//
+// A (activations) and B (weights, rows = output features) are K-major bf16 in
+// global memory, streamed by TMA into 128-byte-swizzled shared-memory stages.
+// One thread issues tcgen05.mma (M=128, N=BN, K=16 per instruction) into a
+// double-buffered fp32 accumulator in tensor memory; four epilogue warps read
+// it back with tcgen05.ld and apply the fused epilogue:
+//   kStoreF32   C = acc                         (fp32)
+//   kAddF32     C += acc                        (fp32 residual stream)
+//   kAtomicF32  C += acc with atomics           (split-K partial sums)
+//   kStoreBF16  C = bf16(acc)
+//   kSwiGLU     B rows are interleaved in blocks of 64 (gate, up); the
+//               output is bf16(silu(gate) * up) with N/2 columns.
+// The kernel is persistent: gridDim.x CTAs walk the tile list (grouped along
+// M so that concurrently running CTAs share A and B tiles in L2).
+#pragma once
+
+#include "ptx.cuh"
+
+namespace gf {
+
+enum GemmMode { kStoreF32 = 0, kAddF32 = 1, kAtomicF32 = 2, kStoreBF16 = 3, kSwiGLU = 4 };
+
+struct GemmArgs {
+  int M, N, K;
+  int num_m, num_n, splits;
+  int kb_total, kb_per_split;
+  int group_m;
+  void* out;
+  int64_t ldo;  // elements
+  int* err;
+};
+
+template <int BN>
+struct GemmCfg {
+  static constexpr int BM = 128;
+  static constexpr int BK = 64;
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
+  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulator buffers (128, 256 or 512 columns)
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+  static constexpr int THREADS = 192;
+};
+
+__device__ __forceinline__ void gemm_tile_coords(const GemmArgs& p, int tile, int& m_blk, int& n_blk, int& split) {
+  split = tile % p.splits;
+  const int t = tile / p.splits;
+  const int group_size = p.group_m * p.num_n;
+  const int g = t / group_size;
+  const int first_m = g * p.group_m;
+  const int gm = min(p.num_m - first_m, p.group_m);
+  const int in = t % group_size;
+  m_blk = first_m + in % gm;
+  n_blk = in / gm;
+}
+
+template <int MODE>
+__device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& p, int row, int col, const uint32_t (&r)[32]) {
+  if (MODE == kStoreF32) {
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + col);
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      dst[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]), __uint_as_float(r[4 * i + 2]),
+                           __uint_as_float(r[4 * i + 3]));
+  } else if (MODE == kAddF32) {
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + col);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      float4 o = dst[i];
+      o.x += __uint_as_float(r[4 * i]);
+      o.y += __uint_as_float(r[4 * i + 1]);
+      o.z += __uint_as_float(r[4 * i + 2]);
+      o.w += __uint_as_float(r[4 * i + 3]);
+      dst[i] = o;
+    }
+  } else if (MODE == kAtomicF32) {
+    float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + col);
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      atomicAdd(dst + i, make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]),
+                                     __uint_as_float(r[4 * i + 2]), __uint_as_float(r[4 * i + 3])));
+  } else if (MODE == kStoreBF16) {
+    uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + (int64_t)row * p.ldo + col);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      uint4 v;
+      v.x = pack_bf16(__uint_as_float(r[8 * i + 0]), __uint_as_float(r[8 * i + 1]));
+      v.y = pack_bf16(__uint_as_float(r[8 * i + 2]), __uint_as_float(r[8 * i + 3]));
+      v.z = pack_bf16(__uint_as_float(r[8 * i + 4]), __uint_as_float(r[8 * i + 5]));
+      v.w = pack_bf16(__uint_as_float(r[8 * i + 6]), __uint_as_float(r[8 * i + 7]));
+      dst[i] = v;
+    }
+  }
+}
+
+template <int BN, int MODE>
+__global__ void __launch_bounds__(192, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const GemmArgs p) {
+  using C = GemmCfg<BN>;
+  constexpr uint32_t IDESC = idesc_bf16_f32(C::BM, BN);
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* acc_full = empty + C::STAGES;
+  uint64_t* acc_empty = acc_full + 2;
+  uint64_t* mma_done = acc_empty + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&acc_full[a], 1);
+      mbar_init(&acc_empty[a], 128);
+    }
+    mbar_init(mma_done, 1);
+    fence_mbar_init();
+    fence_async_smem();
+    prefetch_tmap(&tmA);
+    prefetch_tmap(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+  const int num_tiles = p.num_m * p.num_n * p.splits;
+
+  if (warp == 0) {
+    // ------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int issued = 0;
+      bool ok = true;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        int m_blk, n_blk, split;
+        gemm_tile_coords(p, tile, m_blk, n_blk, split);
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&empty[stage], phase ^ 1u, p.err)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+          tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
+          tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
+          ++issued;
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
+      // Every copy this thread started must have landed before the CTA exits.
+      const int outstanding = min(issued, C::STAGES);
+      for (int i = 0; i < outstanding; ++i) {
+        if (--stage < 0) {
+          stage = C::STAGES - 1;
+          phase ^= 1u;
+        }
+        mbar_wait_drain(&full[stage], phase);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      int acc = 0;
+      uint32_t acc_phase = 0;
+      bool ok = true;
+      bool any = false;
+      for (int tile = blockIdx.x; tile < num_tiles && ok; tile += gridDim.x) {
+        int m_blk, n_blk, split;
+        gemm_tile_coords(p, tile, m_blk, n_blk, split);
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
+        if (!mbar_wait(&acc_empty[acc], acc_phase ^ 1u, p.err)) break;
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        for (int kb = kb0; kb < kb1; ++kb) {
+          if (!mbar_wait(&full[stage], phase, p.err)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a0 = smem_u32(sA + stage * C::A_BYTES);
+          const uint32_t b0 = smem_u32(sB + stage * C::B_BYTES);
+#pragma unroll
+          for (int k = 0; k < C::BK / 16; ++k) {
+            umma_bf16(d_tmem, sdesc_k_sw128(a0 + k * 32), sdesc_k_sw128(b0 + k * 32), IDESC,
+                      (kb > kb0 || k > 0) ? 1u : 0u);
+          }
+          umma_commit(&empty[stage]);
+          any = true;
+          if (++stage == C::STAGES) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        umma_commit(&acc_full[acc]);
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      // All MMAs must be complete before tensor memory is released.
+      if (any) {
+        umma_commit(mma_done);
+        mbar_wait_drain(mma_done, 0);
+      }
+    }
+  } else {
+    // ------------------------------------------------ epilogue (warps 2..5)
+    const int quarter = warp & 3;  // tensor-memory lanes this warp may read
+    const int row_in_tile = quarter * 32 + lane;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
+      int m_blk, n_blk, split;
+      gemm_tile_coords(p, tile, m_blk, n_blk, split);
+      if (!mbar_wait(&acc_full[acc], acc_phase, p.err)) break;
+      tc_fence_after();
+      const int row = m_blk * C::BM + row_in_tile;
+      const bool row_ok = row < p.M;
+      const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
+      if (MODE == kSwiGLU) {
+#pragma unroll 1
+        for (int g = 0; g < BN / 128; ++g) {
+#pragma unroll 1
+          for (int h = 0; h < 2; ++h) {
+            uint32_t rg[32], ru[32];
+            tmem_ld32(taddr + g * 128 + h * 32, rg);
+            tmem_ld32(taddr + g * 128 + 64 + h * 32, ru);
+            tmem_ld_wait();
+            const int gate_col = n_blk * BN + g * 128 + h * 32;
+            if (row_ok && gate_col < p.N) {
+              const int out_col = n_blk * (BN / 2) + g * 64 + h * 32;
+              uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) +
+                                                    (int64_t)row * p.ldo + out_col);
+#pragma unroll
+              for (int i = 0; i < 4; ++i) {
+                float o[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                  const float gv = __uint_as_float(rg[8 * i + j]);
+                  const float uv = __uint_as_float(ru[8 * i + j]);
+                  o[j] = gv / (1.0f + __expf(-gv)) * uv;
+                }
+                uint4 v;
+                v.x = pack_bf16(o[0], o[1]);
+                v.y = pack_bf16(o[2], o[3]);
+                v.z = pack_bf16(o[4], o[5]);
+                v.w = pack_bf16(o[6], o[7]);
+                dst[i] = v;
+              }
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c, r);
+          tmem_ld_wait();
+          const int col = n_blk * BN + c;
+          if (row_ok && col < p.N) gemm_epilogue_chunk<MODE>(p, row, col, r);
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&acc_empty[acc]);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, C::TMEM_COLS);
+  }
+}
+
+}  // namespace gf

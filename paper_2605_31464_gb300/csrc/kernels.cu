@@ -1,0 +1,371 @@
+// Memory-bound kernels of the forward pass: embedding gather, RMSNorm,
+// rotary embedding with the paged KV-cache write, greedy arg max, the verdict
+// (restricted softmax, confidence, defer), and bookkeeping.
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace gf {
+
+// ------------------------------------------------------------------ embedding
+// out[t, :] = float(table[ids[t], :]); an id outside [0, vocab) records
+// GF_EINVAL in the error word and yields a zero row.
+__global__ void embed_kernel(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err) {
+  const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (t >= T) return;
+  const int id = ids[t];
+  float* dst = out + (int64_t)t * d;
+  if (id < 0 || id >= vocab) {
+    if (lane == 0) atomicCAS(err, 0, 1);
+    for (int i = lane * 4; i < d; i += 128) *reinterpret_cast<float4*>(dst + i) = make_float4(0.f, 0.f, 0.f, 0.f);
+    return;
+  }
+  const bf16* src = table + (int64_t)id * d;
+  for (int i = lane * 8; i < d; i += 256) {
+    const uint4 v = *reinterpret_cast<const uint4*>(src + i);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
+    float2 f0 = __bfloat1622float2(h[0]), f1 = __bfloat1622float2(h[1]);
+    float2 f2 = __bfloat1622float2(h[2]), f3 = __bfloat1622float2(h[3]);
+    *reinterpret_cast<float4*>(dst + i) = make_float4(f0.x, f0.y, f1.x, f1.y);
+    *reinterpret_cast<float4*>(dst + i + 4) = make_float4(f2.x, f2.y, f3.x, f3.y);
+  }
+}
+
+cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err,
+                         cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  embed_kernel<<<(T + 7) / 8, 256, 0, s>>>(ids, T, table, vocab, d, out, err);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ RMSNorm
+// y[r, :] = bf16(x[src, :] * rsqrt(mean(x[src, :]^2) + eps) * gain), src = row_idx ? row_idx[r] : r.
+__global__ void rmsnorm_kernel(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d,
+                               const float* gain, float eps, bf16* y, int64_t ldy) {
+  const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const int src = row_idx ? row_idx[r] : r;
+  const float* xr = x + (int64_t)src * ldx;
+  float ss = 0.f;
+  for (int i = lane * 4; i < d; i += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + i);
+    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  const float inv = rsqrtf(ss / (float)d + eps);
+  bf16* yr = y + (int64_t)r * ldy;
+  for (int i = lane * 4; i < d; i += 128) {
+    const float4 v = *reinterpret_cast<const float4*>(xr + i);
+    const float4 g = *reinterpret_cast<const float4*>(gain + i);
+    uint2 o;
+    o.x = pack_bf16(v.x * inv * g.x, v.y * inv * g.y);
+    o.y = pack_bf16(v.z * inv * g.z, v.w * inv * g.w);
+    *reinterpret_cast<uint2*>(yr + i) = o;
+  }
+}
+
+cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
+                           float eps, bf16* y, int64_t ldy, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  rmsnorm_kernel<<<(rows + 7) / 8, 256, 0, s>>>(x, ldx, row_idx, rows, d, gain, eps, y, ldy);
+  return cudaGetLastError();
+}
+
+__global__ void last_rows_kernel(const int32_t* offsets, int B, int32_t* row_idx) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) row_idx[b] = offsets[b + 1] - 1;
+}
+cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  last_rows_kernel<<<(B + 255) / 256, 256, 0, s>>>(offsets, B, row_idx);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ RoPE + KV write
+// One block per token.  q and k heads are rotated pairwise (i, i + hd/2) by
+// angle pos * theta^(-2i/hd) (cos/sin from the table), rounded to bf16 and
+// written to the rotated-query buffer or the key cache; v heads are copied
+// to the value cache.  Cache row of (layer, page, kv head, slot-in-page).
+__global__ void rope_kv_kernel(const RopeKvArgs a) {
+  const int t = blockIdx.x;
+  int slot, pos;
+  if (a.offsets) {
+    int lo = 0, hi = a.B - 1;  // item with offsets[item] <= t < offsets[item+1]
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.offsets[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    slot = a.slots[lo];
+    pos = t - a.offsets[lo];
+  } else {
+    slot = a.handles[t];
+    pos = a.seq_len[slot];
+  }
+  const int half = a.hd / 2;
+  const int heads = a.n_q + 2 * a.n_kv;
+  const int page = a.block_table[(int64_t)slot * a.max_pages + (pos >> 6)];
+  const int in_page = pos & 63;
+  float* src = a.qkv + (int64_t)t * a.ldqkv;
+  const float2* cs = a.rope_cs + (int64_t)pos * half;
+  for (int idx = threadIdx.x; idx < heads * half; idx += blockDim.x) {
+    const int h = idx / half, i = idx % half;
+    const int c0 = h * a.hd + i;
+    const float x0 = src[c0], x1 = src[c0 + half];
+    if (a.zero_after) {
+      src[c0] = 0.f;
+      src[c0 + half] = 0.f;
+    }
+    if (h < a.n_q + a.n_kv) {
+      const float2 r = cs[i];
+      const bf16 y0 = __float2bfloat16(x0 * r.x - x1 * r.y);
+      const bf16 y1 = __float2bfloat16(x1 * r.x + x0 * r.y);
+      if (h < a.n_q) {
+        bf16* dst = a.q_out + (int64_t)t * a.ldq + h * a.hd;
+        dst[i] = y0;
+        dst[i + half] = y1;
+      } else {
+        const int g = h - a.n_q;
+        bf16* dst = a.k_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + g) * 64 + in_page) * a.hd;
+        dst[i] = y0;
+        dst[i + half] = y1;
+      }
+    } else {
+      const int g = h - a.n_q - a.n_kv;
+      bf16* dst = a.v_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + g) * 64 + in_page) * a.hd;
+      dst[i] = __float2bfloat16(x0);
+      dst[i + half] = __float2bfloat16(x1);
+    }
+  }
+}
+
+cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s) {
+  if (a.T <= 0) return cudaSuccess;
+  rope_kv_kernel<<<a.T, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+// (cos, sin) of pos * theta^(-2i/hd), evaluated in double precision.
+__global__ void rope_table_kernel(double theta, int hd, int max_seq, float2* cs) {
+  const int half = hd / 2;
+  const int64_t n = (int64_t)max_seq * half;
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x) {
+    const int pos = (int)(k / half), i = (int)(k % half);
+    const double inv_freq = pow(theta, -2.0 * i / (double)hd);
+    double sn, cn;
+    sincos((double)pos * inv_freq, &sn, &cn);
+    cs[k] = make_float2((float)cn, (float)sn);
+  }
+}
+cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cudaStream_t s) {
+  rope_table_kernel<<<1024, 256, 0, s>>>((double)theta, hd, max_seq, cs);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ greedy arg max
+// out[b] = arg max_v logits[b, v], lowest v on ties; optionally also out2[b*stride].
+__global__ void argmax_kernel(const float* logits, int64_t ld, int V, int32_t* out, int32_t* out2,
+                              int64_t out2_stride) {
+  const int b = blockIdx.x;
+  const float* row = logits + (int64_t)b * ld;
+  float best = -INFINITY;
+  int best_i = 0x7fffffff;
+  for (int i = threadIdx.x; i < V; i += blockDim.x) {
+    const float v = row[i];
+    if (v > best || (v == best && i < best_i)) {
+      best = v;
+      best_i = i;
+    }
+  }
+  __shared__ float sv[32];
+  __shared__ int si[32];
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, best_i, o);
+    if (ov > best || (ov == best && oi < best_i)) {
+      best = ov;
+      best_i = oi;
+    }
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) {
+    sv[warp] = best;
+    si[warp] = best_i;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int nw = blockDim.x >> 5;
+    best = lane < nw ? sv[lane] : -INFINITY;
+    best_i = lane < nw ? si[lane] : 0x7fffffff;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, best, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, best_i, o);
+      if (ov > best || (ov == best && oi < best_i)) {
+        best = ov;
+        best_i = oi;
+      }
+    }
+    if (lane == 0) {
+      if (best_i == 0x7fffffff) best_i = 0;  // all NaN: fall back to id 0
+      out[b] = best_i;
+      if (out2) out2[(int64_t)b * out2_stride] = best_i;
+    }
+  }
+}
+cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
+                          int64_t out2_stride, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  argmax_kernel<<<B, 1024, 0, s>>>(logits, ld, V, out, out2, out2_stride);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ verdict (Sec. 2.1)
+// p = softmax(logits[b, ids]); conf = max p; arg = first arg max; defer = conf < tau.
+struct VerdictIds {
+  int32_t v[8];
+};
+__global__ void verdict_kernel(const float* logits, int64_t ld, int B, VerdictIds ids, int K, float tau, float* p,
+                               float* conf, int32_t* arg, uint8_t* defer) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= B) return;
+  const float* row = logits + (int64_t)b * ld;
+  float z[8];
+  float mx = -INFINITY;
+  for (int k = 0; k < K; ++k) {
+    z[k] = row[ids.v[k]];
+    mx = fmaxf(mx, z[k]);
+  }
+  float sum = 0.f;
+  for (int k = 0; k < K; ++k) {
+    z[k] = expf(z[k] - mx);
+    sum += z[k];
+  }
+  float best = -1.f;
+  int best_k = 0;
+  for (int k = 0; k < K; ++k) {
+    const float pk = z[k] / sum;
+    p[(int64_t)b * K + k] = pk;
+    if (pk > best) {
+      best = pk;
+      best_k = k;
+    }
+  }
+  conf[b] = best;
+  arg[b] = best_k;
+  defer[b] = best < tau ? 1 : 0;
+}
+cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t* ids, int K, float tau, float* p,
+                           float* conf, int32_t* arg, uint8_t* defer, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  VerdictIds v;
+  for (int k = 0; k < 8; ++k) v.v[k] = k < K ? ids[k] : 0;
+  verdict_kernel<<<(B + 127) / 128, 128, 0, s>>>(logits, ld, B, v, K, tau, p, conf, arg, defer);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ bookkeeping
+__global__ void set_seq_len_kernel(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) seq_len[slots[b]] = offsets[b + 1] - offsets[b];
+}
+cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
+                               cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  set_seq_len_kernel<<<(B + 255) / 256, 256, 0, s>>>(offsets, slots, B, seq_len);
+  return cudaGetLastError();
+}
+
+__global__ void advance_kernel(const int32_t* handles, int B, int32_t* seq_len) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b < B) seq_len[handles[b]] += 1;
+}
+cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(handles, B, seq_len);
+  return cudaGetLastError();
+}
+
+// prompt_b = inc_ids[inc_off[b]:inc_off[b+1]] ++ cand_ids[cand_off[b]:cand_off[b+1]], packed at prompt_off[b].
+__global__ void build_prompts_kernel(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
+                                     const int32_t* cand_off, const int32_t* prompt_off, int B, int T,
+                                     int32_t* out) {
+  for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x) {
+    int lo = 0, hi = B - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (prompt_off[mid] <= t) lo = mid; else hi = mid - 1;
+    }
+    const int j = t - prompt_off[lo];
+    const int n_inc = inc_off[lo + 1] - inc_off[lo];
+    out[t] = j < n_inc ? inc_ids[inc_off[lo] + j] : cand_ids[cand_off[lo] + (j - n_inc)];
+  }
+}
+cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
+                                 const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
+                                 cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  int blocks = (T + 255) / 256;
+  if (blocks > 4096) blocks = 4096;
+  build_prompts_kernel<<<blocks, 256, 0, s>>>(inc_ids, inc_off, cand_ids, cand_off, prompt_off, B, T, out);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ weight packing
+// dst rows [128c, 128c+64) = gate rows [64c, 64c+64), dst rows [128c+64, 128c+128) = up rows;
+// rows past F are zero.  Fp = F rounded up to 64.
+__global__ void pack_gate_up_kernel(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst) {
+  const int64_t chunks_per_row = d / 8;
+  const int64_t n = (int64_t)2 * Fp * chunks_per_row;
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t r = k / chunks_per_row, c = k % chunks_per_row;
+    const int64_t blk = r / 128, in = r % 128;
+    const bool is_up = in >= 64;
+    const int64_t f = blk * 64 + (in & 63);
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (f < F) v = *reinterpret_cast<const uint4*>((is_up ? up : gate) + f * d + c * 8);
+    *reinterpret_cast<uint4*>(dst + r * d + c * 8) = v;
+  }
+}
+cudaError_t launch_pack_gate_up(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst, cudaStream_t s) {
+  pack_gate_up_kernel<<<2048, 256, 0, s>>>(gate, up, F, Fp, d, dst);
+  return cudaGetLastError();
+}
+
+__global__ void bf16_to_f32_kernel(const bf16* src, int64_t n, float* dst) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x)
+    dst[k] = __bfloat162float(src[k]);
+}
+cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStream_t s) {
+  bf16_to_f32_kernel<<<256, 256, 0, s>>>(src, n, dst);
+  return cudaGetLastError();
+}
+
+// ------------------------------------------------------------------ inspection
+__global__ void read_kv_kernel(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,
+                               int slot, int start, int n, int n_kv, int hd, int64_t layer_row0, bf16* k_dst,
+                               bf16* v_dst) {
+  const int64_t total = (int64_t)n * n_kv * hd;
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < total; k += (int64_t)gridDim.x * blockDim.x) {
+    const int i = (int)(k % hd);
+    const int g = (int)((k / hd) % n_kv);
+    const int t = (int)(k / ((int64_t)hd * n_kv));
+    const int pos = start + t;
+    const int page = block_table[(int64_t)slot * max_pages + (pos >> 6)];
+    const int64_t src = (layer_row0 + ((int64_t)page * n_kv + g) * 64 + (pos & 63)) * hd + i;
+    k_dst[k] = k_cache[src];
+    v_dst[k] = v_cache[src];
+  }
+}
+cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,
+                           int slot, int start, int n, int n_kv, int hd, int64_t layer_row0, bf16* k_dst,
+                           bf16* v_dst, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  read_kv_kernel<<<1024, 256, 0, s>>>(k_cache, v_cache, block_table, max_pages, slot, start, n, n_kv, hd, layer_row0,
+                                      k_dst, v_dst);
+  return cudaGetLastError();
+}
+
+}  // namespace gf

@@ -1,0 +1,104 @@
+// Kernel argument structs and launch wrappers shared by the runtime.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace gf {
+
+using bf16 = __nv_bfloat16;
+
+// ------------------------------------------------------------------ GEMM
+// C[M,N] (op)= A[M,K] . B[N,K]^T ; mode is a GemmMode.  tmA/tmB are 2D
+// tensor maps (bf16, 128-byte swizzle) with boxes {64, 128} and {64, bn}.
+int gemm_num_stages(int bn);
+int gemm_smem_bytes(int bn);
+cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
+                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s);
+
+// ------------------------------------------------------------------ attention
+struct PrefillAttnArgs {
+  const int2* items;          // (item, q_tile) work list, heaviest first
+  const int32_t* offsets;     // [B+1] token offsets of the packed prompts
+  const int32_t* slots;       // [B] sequence slot of each prompt
+  const int32_t* block_table; // [slots][max_pages]
+  int max_pages;
+  int n_q, n_kv;
+  int64_t layer_row0;         // first cache row of this layer: layer * num_pages * n_kv * 64
+  bf16* out;                  // [T, n_q*hd]
+  int64_t ldo;
+  float scale_log2;           // log2(e) / sqrt(hd)
+  int* err;
+};
+cudaError_t launch_attn_prefill(int hd, const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
+                                const PrefillAttnArgs& a, int n_items, cudaStream_t s);
+
+struct DecodeAttnArgs {
+  const bf16* q;              // [B, n_q*hd], rotated queries of this step
+  int64_t ldq;
+  const int32_t* handles;     // [B] slots
+  const int32_t* seq_len;     // [slots] tokens cached before this step; context = seq_len + 1
+  const int32_t* block_table;
+  int max_pages;
+  int n_q, n_kv;
+  int64_t layer_row0;
+  int chunk;                  // keys per split, multiple of 64
+  int max_splits;
+  float* part_o;              // [B][n_kv][max_splits][16][hd] unnormalised partial outputs
+  float* part_ml;             // [B][n_kv][max_splits][16][2] (running max in log2 units, sum)
+  bf16* out;                  // [B, n_q*hd]
+  int64_t ldo;
+  float scale_log2;
+  int* err;
+};
+cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a,
+                               int B, cudaStream_t s);
+
+// ------------------------------------------------------------------ elementwise / small kernels
+struct RopeKvArgs {
+  float* qkv;                 // [T, (n_q+2n_kv)*hd] fp32 projections
+  int64_t ldqkv;
+  bf16* q_out;                // [T, n_q*hd]
+  int64_t ldq;
+  bf16* k_cache;
+  bf16* v_cache;
+  const float2* rope_cs;      // [max_seq][hd/2] (cos, sin)
+  // prefill: offsets/slots describe the packed prompts; decode: offsets == nullptr
+  const int32_t* offsets;
+  const int32_t* slots;
+  int B;
+  const int32_t* handles;
+  const int32_t* seq_len;
+  const int32_t* block_table;
+  int max_pages;
+  int T, n_q, n_kv, hd;
+  int64_t layer_row0;
+  int zero_after;             // write zeros back into qkv after reading (split-K accumulators)
+};
+cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s);
+
+cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err,
+                         cudaStream_t s);
+cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
+                           float eps, bf16* y, int64_t ldy, cudaStream_t s);
+cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s);
+cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
+                          int64_t out2_stride, cudaStream_t s);
+cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t* ids, int K, float tau, float* p,
+                           float* conf, int32_t* arg, uint8_t* defer, cudaStream_t s);
+cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
+                               cudaStream_t s);
+cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s);
+cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
+                                 const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
+                                 cudaStream_t s);
+cudaError_t launch_pack_gate_up(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst, cudaStream_t s);
+cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStream_t s);
+cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cudaStream_t s);
+cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,
+                           int slot, int start, int n, int n_kv, int hd, int64_t layer_row0, bf16* k_dst,
+                           bf16* v_dst, cudaStream_t s);
+
+}  // namespace gf

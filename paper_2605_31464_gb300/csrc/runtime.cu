@@ -1,0 +1,1035 @@
+// Host runtime behind the C ABI (include/gf.h): model creation and weight
+// packing, the paged KV pool and its block tables, and the orchestration of
+// prefill, greedy decode and the verdict/defer step on one CUDA stream.
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <tuple>
+#include <vector>
+
+#include "gf.h"
+#include "gemm_tc.cuh"
+#include "kernels.h"
+
+using gf::bf16;
+
+namespace {
+
+thread_local std::string g_err = "no error";
+
+int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+#define CU(x)                                                                                          \
+  do {                                                                                                 \
+    cudaError_t e_ = (x);                                                                              \
+    if (e_ != cudaSuccess)                                                                             \
+      return fail(GF_ECUDA, "%s failed: %s (%s:%d)", #x, cudaGetErrorString(e_), __FILE__, __LINE__); \
+  } while (0)
+
+#define TRY(x)             \
+  do {                     \
+    int rc_ = (x);         \
+    if (rc_ != GF_OK) return rc_; \
+  } while (0)
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 2D bf16 tensor map: `outer` rows of `inner` elements, row pitch in bytes,
+// box {box_inner, box_outer}, 128-byte swizzle, zero fill out of bounds.
+int make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+             uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return fail(GF_ECUDA, "cuTensorMapEncodeTiled is unavailable");
+  cuuint64_t dims[2] = {inner, outer};
+  cuuint64_t strides[1] = {pitch_bytes};
+  cuuint32_t box[2] = {box_inner, box_outer};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS)
+    return fail(GF_ECUDA, "cuTensorMapEncodeTiled failed (%d): inner %llu outer %llu pitch %llu box %u x %u",
+                (int)r, (unsigned long long)inner, (unsigned long long)outer, (unsigned long long)pitch_bytes,
+                box_inner, box_outer);
+  return GF_OK;
+}
+
+// Pinned staging buffers for host->device uploads; a slot is reused only
+// after the copy that last read it has executed.
+struct Staging {
+  struct Slot {
+    void* host = nullptr;
+    size_t cap = 0;
+    cudaEvent_t ev = nullptr;
+  };
+  std::vector<Slot> slots;
+  size_t next = 0;
+  void release() {
+    for (auto& s : slots) {
+      if (s.ev) {
+        cudaEventSynchronize(s.ev);
+        cudaEventDestroy(s.ev);
+      }
+      if (s.host) cudaFreeHost(s.host);
+    }
+    slots.clear();
+  }
+};
+
+int upload(Staging& st, void* dst, const void* src, size_t bytes, cudaStream_t s) {
+  if (bytes == 0) return GF_OK;
+  if (st.slots.empty()) st.slots.resize(8);
+  Staging::Slot& sl = st.slots[st.next];
+  st.next = (st.next + 1) % st.slots.size();
+  if (!sl.ev) CU(cudaEventCreateWithFlags(&sl.ev, cudaEventDisableTiming));
+  CU(cudaEventSynchronize(sl.ev));
+  if (sl.cap < bytes) {
+    if (sl.host) CU(cudaFreeHost(sl.host));
+    sl.host = nullptr;
+    sl.cap = 0;
+    size_t cap = std::max<size_t>(bytes, 1 << 16);
+    if (cudaHostAlloc(&sl.host, cap, cudaHostAllocDefault) != cudaSuccess) return fail(GF_ENOMEM, "pinned staging");
+    sl.cap = cap;
+  }
+  memcpy(sl.host, src, bytes);
+  CU(cudaMemcpyAsync(dst, sl.host, bytes, cudaMemcpyHostToDevice, s));
+  CU(cudaEventRecord(sl.ev, s));
+  return GF_OK;
+}
+
+struct Capture {
+  int layer, item;
+  float* dst;
+  int64_t cap;
+};
+
+}  // namespace
+
+struct gf_model {
+  gf_config cfg{};
+  int dev = 0, sms = 0;
+  int L = 0, d = 0, nq = 0, nkv = 0, hd = 0, ffn = 0, ffn_pad = 0, vocab = 0, qkv_dim = 0, q_dim = 0;
+  int64_t num_pages = 0;
+  int max_pages = 0;  // pages per sequence
+  int64_t T_max = 0;
+  int B_max = 0;
+
+  std::vector<void*> allocs;
+  struct Layer {
+    bf16 *qkv = nullptr, *o = nullptr, *gu = nullptr, *down = nullptr;
+    float *attn_norm = nullptr, *ffn_norm = nullptr;
+  };
+  std::vector<Layer> layers;
+  bf16 *embed = nullptr, *head = nullptr;
+  float* final_norm = nullptr;
+  bf16 *k_cache = nullptr, *v_cache = nullptr;
+  CUtensorMap tm_k{}, tm_v{};
+  int32_t *bt = nullptr, *seq_len = nullptr;
+  float2* rope_cs = nullptr;
+
+  // prefill activations (T_max rows)
+  float* resid = nullptr;
+  bf16* xn = nullptr;
+  float* qkv = nullptr;
+  bf16* q = nullptr;
+  bf16* attn = nullptr;
+  bf16* act = nullptr;
+  int32_t* prompt_ids = nullptr;
+  int32_t* in_ids = nullptr;
+  // small activations (B_max rows)
+  float* dres = nullptr;
+  bf16* dxn = nullptr;
+  float* dqkv = nullptr;
+  bf16* dq = nullptr;
+  bf16* dattn = nullptr;
+  bf16* dact = nullptr;
+  float *part_o = nullptr, *part_ml = nullptr;
+  int dec_chunk = 256, dec_max_splits = 1;
+  float* logits = nullptr;  // [B_max, vocab]
+  int32_t* last_idx = nullptr;
+  int32_t* next = nullptr;
+  int32_t* handles = nullptr;  // decode handles
+  int32_t* call = nullptr;     // prefill descriptor: offsets | slots | items
+  size_t call_ints = 0;
+  int32_t* fcall = nullptr;    // forecast descriptor: inc_off | cand_off | prompt_off
+  float* out_small = nullptr;  // host-variant outputs on the device
+  int* err = nullptr;
+
+  // host mirrors
+  std::vector<int32_t> h_bt, h_len;
+  std::vector<char> live;
+  std::vector<int32_t> free_pages, free_slots;
+  std::vector<Capture> caps;
+  std::map<std::tuple<const void*, uint64_t, uint64_t, uint32_t>, CUtensorMap> maps;
+  Staging staging;
+  int64_t launches = 0;
+  // live kernel timing (gf_profile_*)
+  uint32_t prof_mask = 0;
+  struct ProfRec {
+    cudaEvent_t a, b;
+    int kind;
+    double flops, bytes;
+  };
+  std::vector<ProfRec> prof;
+  std::vector<cudaEvent_t> ev_pool;
+  void* host_out = nullptr;
+  size_t host_out_cap = 0;
+};
+
+namespace {
+
+template <typename T>
+int dalloc(gf_model* m, T** p, size_t count) {
+  void* v = nullptr;
+  size_t bytes = std::max<size_t>(count * sizeof(T), 256);
+  if (cudaMalloc(&v, bytes) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(GF_ENOMEM, "cudaMalloc of %zu bytes failed", bytes);
+  }
+  m->allocs.push_back(v);
+  *p = reinterpret_cast<T*>(v);
+  return GF_OK;
+}
+
+int get_map(gf_model* m, const void* base, uint64_t inner, uint64_t outer, uint32_t box_outer, CUtensorMap* out) {
+  auto key = std::make_tuple(base, inner, outer, box_outer);
+  auto it = m->maps.find(key);
+  if (it != m->maps.end()) {
+    *out = it->second;
+    return GF_OK;
+  }
+  TRY(make_map(out, base, inner, outer, inner * 2, 64, box_outer));
+  if (m->maps.size() > 4096) m->maps.clear();
+  m->maps[key] = *out;
+  return GF_OK;
+}
+
+cudaEvent_t pool_event(gf_model* m) {
+  if (!m->ev_pool.empty()) {
+    cudaEvent_t e = m->ev_pool.back();
+    m->ev_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+// Brackets one launch with events when its kernel class is being timed.
+struct ProfScope {
+  gf_model* m;
+  cudaStream_t s;
+  int kind;
+  double flops, bytes;
+  cudaEvent_t a = nullptr;
+  ProfScope(gf_model* m_, cudaStream_t s_, int kind_, double flops_, double bytes_)
+      : m(m_), s(s_), kind(kind_), flops(flops_), bytes(bytes_) {
+    if (m->prof_mask & (1u << kind)) {
+      a = pool_event(m);
+      cudaEventRecord(a, s);
+    }
+  }
+  ~ProfScope() {
+    if (a) {
+      cudaEvent_t b = pool_event(m);
+      cudaEventRecord(b, s);
+      m->prof.push_back({a, b, kind, flops, bytes});
+    }
+  }
+};
+
+// Tile width and split-K factor for a GEMM of M rows.
+void plan_gemm(const gf_model* m, int M, int N, int K, int mode, int* bn, int* splits) {
+  const int num_m = (M + 127) / 128;
+  *splits = 1;
+  if (mode == gf::kSwiGLU) {
+    *bn = num_m >= 4 ? 256 : 128;
+    return;
+  }
+  if (num_m >= 4) {
+    *bn = 256;
+    return;
+  }
+  if (mode != gf::kAtomicF32) {
+    *bn = 128;
+    return;
+  }
+  *bn = 64;
+  const int tiles = num_m * ((N + 63) / 64);
+  const int kb = K / 64;
+  int s = (2 * m->sms + tiles - 1) / tiles;
+  s = std::min(s, std::max(1, kb / 4));
+  *splits = std::max(1, s);
+}
+
+// n_alg / k_alg: the unpadded output width and contraction length (algorithmic work).
+int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
+         cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0) {
+  if (M <= 0) return GF_OK;
+  int bn, splits;
+  plan_gemm(m, M, N, K, mode, &bn, &splits);
+  CUtensorMap ta, tb;
+  TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, 128, &ta));
+  TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, (uint32_t)bn, &tb));
+  const double na = n_alg ? n_alg : N, ka = k_alg ? k_alg : K;
+  const double out_bytes = (mode == gf::kSwiGLU ? na / 2 * 2 : na * (mode == gf::kStoreBF16 ? 2 : 4)) * M;
+  ProfScope ps(m, s, decode ? GF_PROF_DECODE_GEMM : GF_PROF_PREFILL_GEMM, 2.0 * M * na * ka,
+               na * ka * 2 + (double)M * ka * 2 + out_bytes * (mode == gf::kAddF32 || mode == gf::kAtomicF32 ? 2 : 1));
+  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
+  m->launches += 1;
+  return GF_OK;
+}
+
+int64_t layer_row0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * 64; }
+
+
+
+int fire_captures(gf_model* m, int layer, const float* base, const int32_t* offsets_host, int B, bool decode,
+                  cudaStream_t s) {
+  for (size_t i = 0; i < m->caps.size();) {
+    Capture& c = m->caps[i];
+    if (c.layer == layer && c.item < B) {
+      int64_t row0 = decode ? c.item : offsets_host[c.item];
+      int64_t rows = decode ? 1 : (offsets_host[c.item + 1] - offsets_host[c.item]);
+      rows = std::min(rows, c.cap);
+      CU(cudaMemcpyAsync(c.dst, base + row0 * m->d, rows * m->d * sizeof(float), cudaMemcpyDeviceToDevice, s));
+      m->caps.erase(m->caps.begin() + i);
+    } else {
+      ++i;
+    }
+  }
+  return GF_OK;
+}
+
+int alloc_pages(gf_model* m, int slot, int first, int count, std::vector<std::pair<int, int>>* undo) {
+  for (int j = first; j < first + count; ++j) {
+    if (m->h_bt[(int64_t)slot * m->max_pages + j] >= 0) continue;
+    if (m->free_pages.empty()) return fail(GF_ECAPACITY, "KV page pool exhausted");
+    const int p = m->free_pages.back();
+    m->free_pages.pop_back();
+    m->h_bt[(int64_t)slot * m->max_pages + j] = p;
+    undo->push_back({slot, j});
+  }
+  return GF_OK;
+}
+
+void undo_pages(gf_model* m, const std::vector<std::pair<int, int>>& undo) {
+  for (auto it = undo.rbegin(); it != undo.rend(); ++it) {
+    int32_t& e = m->h_bt[(int64_t)it->first * m->max_pages + it->second];
+    m->free_pages.push_back(e);
+    e = -1;
+  }
+}
+
+void release_slot(gf_model* m, int slot) {
+  for (int j = 0; j < m->max_pages; ++j) {
+    int32_t& e = m->h_bt[(int64_t)slot * m->max_pages + j];
+    if (e >= 0) m->free_pages.push_back(e);
+    e = -1;
+  }
+  m->h_len[slot] = 0;
+  m->live[slot] = 0;
+  m->free_slots.push_back(slot);
+}
+
+int upload_block_table(gf_model* m, cudaStream_t s) {
+  return upload(m->staging, m->bt, m->h_bt.data(), m->h_bt.size() * sizeof(int32_t), s);
+}
+
+// Prefill of B packed prompts already on the device.  `reserve` extra
+// tokens of KV pages are allocated per sequence (decode steps to come).
+int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets, int reserve, int32_t* handles_out,
+                 float* logits_dst, int32_t* next_dst, cudaStream_t s, int32_t* tokens_col = nullptr,
+                 int64_t tokens_stride = 0) {
+  if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
+  if (!ids || !offsets) return fail(GF_EINVAL, "null ids or offsets");
+  if (offsets[0] != 0) return fail(GF_EINVAL, "offsets[0] must be 0");
+  for (int b = 0; b < B; ++b) {
+    const int len = offsets[b + 1] - offsets[b];
+    if (len < 1) return fail(GF_EINVAL, "prompt %d has length %d", b, len);
+    if (len + reserve > m->cfg.max_seq)
+      return fail(GF_ECAPACITY, "prompt %d: %d tokens (+%d) exceed max_seq %d", b, len, reserve, m->cfg.max_seq);
+  }
+  const int64_t T = offsets[B];
+  if (T > m->T_max) return fail(GF_ECAPACITY, "%lld prompt tokens exceed max_prefill_tokens %lld", (long long)T,
+                                (long long)m->T_max);
+  if ((int)m->free_slots.size() < B) return fail(GF_ECAPACITY, "no free sequence slots");
+  // slots and pages
+  std::vector<int32_t> slots(B);
+  std::vector<std::pair<int, int>> undo;
+  for (int b = 0; b < B; ++b) {
+    slots[b] = m->free_slots.back();
+    m->free_slots.pop_back();
+  }
+  for (int b = 0; b < B; ++b) {
+    const int len = offsets[b + 1] - offsets[b];
+    const int rc = alloc_pages(m, slots[b], 0, (len + reserve + 63) / 64, &undo);
+    if (rc != GF_OK) {
+      undo_pages(m, undo);
+      for (int bb = B - 1; bb >= 0; --bb) m->free_slots.push_back(slots[bb]);
+      return rc;
+    }
+  }
+  for (int b = 0; b < B; ++b) {
+    m->live[slots[b]] = 1;
+    m->h_len[slots[b]] = offsets[b + 1] - offsets[b];
+    handles_out[b] = slots[b];
+  }
+  // descriptor: offsets | slots | work items (heaviest first)
+  std::vector<int32_t> desc;
+  desc.insert(desc.end(), offsets, offsets + B + 1);
+  desc.insert(desc.end(), slots.begin(), slots.end());
+  const size_t items_at = desc.size() + (desc.size() & 1);  // int2 alignment
+  desc.resize(items_at);
+  std::vector<std::pair<int, int>> items;
+  for (int b = 0; b < B; ++b) {
+    const int len = offsets[b + 1] - offsets[b];
+    for (int qt = 0; qt < (len + 127) / 128; ++qt) items.push_back({b, qt});
+  }
+  std::stable_sort(items.begin(), items.end(), [&](const std::pair<int, int>& x, const std::pair<int, int>& y) {
+    auto cost = [&](const std::pair<int, int>& it) {
+      const int len = offsets[it.first + 1] - offsets[it.first];
+      return std::min(it.second * 128 + 128, len);
+    };
+    return cost(x) > cost(y);
+  });
+  for (auto& it : items) {
+    desc.push_back(it.first);
+    desc.push_back(it.second);
+  }
+  if (desc.size() > m->call_ints) return fail(GF_ECAPACITY, "prefill descriptor too large");
+  TRY(upload(m->staging, m->call, desc.data(), desc.size() * sizeof(int32_t), s));
+  TRY(upload_block_table(m, s));
+  const int32_t* d_off = m->call;
+  const int32_t* d_slots = m->call + B + 1;
+  const int2* d_items = reinterpret_cast<const int2*>(m->call + items_at);
+
+  CU(gf::launch_embed(ids, (int)T, m->embed, m->vocab, m->d, m->resid, m->err, s));
+  m->launches++;
+  CUtensorMap tq;
+  TRY(get_map(m, m->q, (uint64_t)m->q_dim, (uint64_t)T, 128, &tq));
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)m->hd);
+  for (int l = 0; l < m->L; ++l) {
+    const gf_model::Layer& W = m->layers[l];
+    TRY(fire_captures(m, l, m->resid, offsets, B, false, s));
+    CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.attn_norm, m->cfg.rms_eps, m->xn, m->d, s));
+    m->launches++;
+    TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, m->qkv, m->qkv_dim, gf::kStoreF32, s, false));
+    gf::RopeKvArgs ra{};
+    ra.qkv = m->qkv;
+    ra.ldqkv = m->qkv_dim;
+    ra.q_out = m->q;
+    ra.ldq = m->q_dim;
+    ra.k_cache = m->k_cache;
+    ra.v_cache = m->v_cache;
+    ra.rope_cs = m->rope_cs;
+    ra.offsets = d_off;
+    ra.slots = d_slots;
+    ra.B = B;
+    ra.block_table = m->bt;
+    ra.max_pages = m->max_pages;
+    ra.T = (int)T;
+    ra.n_q = m->nq;
+    ra.n_kv = m->nkv;
+    ra.hd = m->hd;
+    ra.layer_row0 = layer_row0(m, l);
+    ra.zero_after = 0;
+    CU(gf::launch_rope_kv(ra, s));
+    m->launches++;
+    gf::PrefillAttnArgs pa{};
+    pa.items = d_items;
+    pa.offsets = d_off;
+    pa.slots = d_slots;
+    pa.block_table = m->bt;
+    pa.max_pages = m->max_pages;
+    pa.n_q = m->nq;
+    pa.n_kv = m->nkv;
+    pa.layer_row0 = layer_row0(m, l);
+    pa.out = m->attn;
+    pa.ldo = m->q_dim;
+    pa.scale_log2 = scale_log2;
+    pa.err = m->err;
+    {
+      double pairs = 0;
+      for (int b = 0; b < B; ++b) {
+        const double n = offsets[b + 1] - offsets[b];
+        pairs += n * (n + 1) / 2;
+      }
+      ProfScope ps(m, s, GF_PROF_PREFILL_ATTN, pairs * m->nq * 4.0 * m->hd,
+                   (double)T * (m->q_dim * 2 + 2 * m->nkv * m->hd * 2 + m->q_dim * 2));
+      CU(gf::launch_attn_prefill(m->hd, tq, m->tm_k, m->tm_v, pa, (int)items.size(), s));
+    }
+    m->launches++;
+    TRY(gemm(m, m->attn, (int)T, m->q_dim, W.o, m->d, m->resid, m->d, gf::kAddF32, s, false));
+    CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.ffn_norm, m->cfg.rms_eps, m->xn, m->d, s));
+    m->launches++;
+    TRY(gemm(m, m->xn, (int)T, m->d, W.gu, 2 * m->ffn_pad, m->act, m->ffn_pad, gf::kSwiGLU, s, false,
+             2 * m->ffn));
+    TRY(gemm(m, m->act, (int)T, m->ffn_pad, W.down, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, m->ffn));
+  }
+  TRY(fire_captures(m, m->L, m->resid, offsets, B, false, s));
+  CU(gf::launch_last_rows(d_off, B, m->last_idx, s));
+  CU(gf::launch_rmsnorm(m->resid, m->d, m->last_idx, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
+  m->launches += 2;
+  float* lg = logits_dst ? logits_dst : m->logits;
+  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, false));
+  if (next_dst) {
+    CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+    m->launches++;
+  }
+  CU(gf::launch_set_seq_len(d_off, d_slots, B, m->seq_len, s));
+  m->launches++;
+  return GF_OK;
+}
+
+// One decode step for B live sequences whose handles are already on the
+// device in m->handles (host copy in `h`).
+int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float* logits_dst, int32_t* next_dst,
+                int32_t* tokens_col, int64_t tokens_stride, cudaStream_t s) {
+  CU(gf::launch_embed(ids, B, m->embed, m->vocab, m->d, m->dres, m->err, s));
+  m->launches++;
+  CU(cudaMemsetAsync(m->dqkv, 0, (size_t)B * m->qkv_dim * sizeof(float), s));
+  const float scale_log2 = 1.4426950408889634f / sqrtf((float)m->hd);
+  for (int l = 0; l < m->L; ++l) {
+    const gf_model::Layer& W = m->layers[l];
+    TRY(fire_captures(m, l, m->dres, nullptr, B, true, s));
+    CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, W.attn_norm, m->cfg.rms_eps, m->dxn, m->d, s));
+    m->launches++;
+    TRY(gemm(m, m->dxn, B, m->d, W.qkv, m->qkv_dim, m->dqkv, m->qkv_dim, gf::kAtomicF32, s, true));
+    gf::RopeKvArgs ra{};
+    ra.qkv = m->dqkv;
+    ra.ldqkv = m->qkv_dim;
+    ra.q_out = m->dq;
+    ra.ldq = m->q_dim;
+    ra.k_cache = m->k_cache;
+    ra.v_cache = m->v_cache;
+    ra.rope_cs = m->rope_cs;
+    ra.offsets = nullptr;
+    ra.handles = m->handles;
+    ra.seq_len = m->seq_len;
+    ra.block_table = m->bt;
+    ra.max_pages = m->max_pages;
+    ra.T = B;
+    ra.n_q = m->nq;
+    ra.n_kv = m->nkv;
+    ra.hd = m->hd;
+    ra.layer_row0 = layer_row0(m, l);
+    ra.zero_after = 1;
+    CU(gf::launch_rope_kv(ra, s));
+    m->launches++;
+    gf::DecodeAttnArgs da{};
+    da.q = m->dq;
+    da.ldq = m->q_dim;
+    da.handles = m->handles;
+    da.seq_len = m->seq_len;
+    da.block_table = m->bt;
+    da.max_pages = m->max_pages;
+    da.n_q = m->nq;
+    da.n_kv = m->nkv;
+    da.layer_row0 = layer_row0(m, l);
+    da.chunk = m->dec_chunk;
+    da.max_splits = m->dec_max_splits;
+    da.part_o = m->part_o;
+    da.part_ml = m->part_ml;
+    da.out = m->dattn;
+    da.ldo = m->q_dim;
+    da.scale_log2 = scale_log2;
+    da.err = m->err;
+    {
+      double ctx = 0;
+      for (int b = 0; b < B; ++b) ctx += m->h_len[h[b]] + 1;
+      ProfScope ps(m, s, GF_PROF_DECODE_ATTN, ctx * m->nq * 4.0 * m->hd,
+                   ctx * 2.0 * m->nkv * m->hd * 2 + (double)B * m->q_dim * 4);
+      CU(gf::launch_attn_decode(m->hd, m->tm_k, m->tm_v, da, B, s));
+    }
+    m->launches += 2;
+    TRY(gemm(m, m->dattn, B, m->q_dim, W.o, m->d, m->dres, m->d, gf::kAtomicF32, s, true));
+    CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, W.ffn_norm, m->cfg.rms_eps, m->dxn, m->d, s));
+    m->launches++;
+    TRY(gemm(m, m->dxn, B, m->d, W.gu, 2 * m->ffn_pad, m->dact, m->ffn_pad, gf::kSwiGLU, s, true, 2 * m->ffn));
+    TRY(gemm(m, m->dact, B, m->ffn_pad, W.down, m->d, m->dres, m->d, gf::kAtomicF32, s, true, 0, m->ffn));
+  }
+  TRY(fire_captures(m, m->L, m->dres, nullptr, B, true, s));
+  CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
+  m->launches++;
+  float* lg = logits_dst ? logits_dst : m->logits;
+  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, true));
+  if (next_dst) {
+    CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+    m->launches++;
+  }
+  CU(gf::launch_advance(m->handles, B, m->seq_len, s));
+  m->launches++;
+  for (int b = 0; b < B; ++b) m->h_len[h[b]] += 1;
+  return GF_OK;
+}
+
+// Validate handles and allocate the pages the next token needs.
+int prepare_decode(gf_model* m, int B, const int32_t* h, cudaStream_t s) {
+  if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
+  std::vector<char> seen(m->B_max, 0);
+  for (int b = 0; b < B; ++b) {
+    if (h[b] < 0 || h[b] >= m->B_max || !m->live[h[b]]) return fail(GF_EINVAL, "handle %d is not live", h[b]);
+    if (seen[h[b]]) return fail(GF_EINVAL, "handle %d repeated", h[b]);
+    seen[h[b]] = 1;
+    if (m->h_len[h[b]] + 1 > m->cfg.max_seq) return fail(GF_ECAPACITY, "sequence %d reached max_seq", h[b]);
+  }
+  std::vector<std::pair<int, int>> undo;
+  for (int b = 0; b < B; ++b) {
+    const int pos = m->h_len[h[b]];
+    const int rc = alloc_pages(m, h[b], pos / 64, 1, &undo);
+    if (rc != GF_OK) {
+      undo_pages(m, undo);
+      return rc;
+    }
+  }
+  if (!undo.empty()) TRY(upload_block_table(m, s));
+  return GF_OK;
+}
+
+}  // namespace
+
+// =====================================================================================================
+// C ABI
+// =====================================================================================================
+extern "C" {
+
+const char* gf_last_error(void) { return g_err.c_str(); }
+
+int64_t gf_launch_count(const gf_model* m) { return m ? m->launches : 0; }
+
+void gf_destroy(gf_model* m) {
+  if (!m) return;
+  cudaDeviceSynchronize();
+  m->staging.release();
+  for (void* p : m->allocs) cudaFree(p);
+  if (m->host_out) cudaFreeHost(m->host_out);
+  delete m;
+}
+
+int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model** out) {
+  if (!cfg || !w || !out) return fail(GF_EINVAL, "null argument");
+  *out = nullptr;
+  const gf_config& c = *cfg;
+  if (c.layers < 1 || c.d_model < 64 || c.d_model % 64 || c.n_q < 1 || c.n_kv < 1 || c.n_q % c.n_kv ||
+      c.ffn < 1 || c.vocab < 32 || c.max_batch < 1 || c.max_batch > 1024 || c.max_seq < 1 ||
+      c.max_prefill_tokens < 1 || !(c.rms_eps >= 0.f) || !(c.rope_theta > 0.f))
+    return fail(GF_EINVAL, "invalid configuration");
+  if (c.head_dim != 64 && c.head_dim != 128) return fail(GF_ENOTIMPL, "head_dim must be 64 or 128");
+  if (c.n_q / c.n_kv > 16) return fail(GF_ENOTIMPL, "more than 16 query heads per KV head");
+  if (c.vocab % 32) return fail(GF_ENOTIMPL, "vocab must be a multiple of 32");
+  if (!w->embed || !w->lm_head || !w->final_norm || !w->attn_norm || !w->wq || !w->wk || !w->wv || !w->wo ||
+      !w->ffn_norm || !w->w_gate || !w->w_up || !w->w_down)
+    return fail(GF_EINVAL, "null weight pointer");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  gf_model* m = new gf_model();
+  m->cfg = c;
+  int rc = GF_OK;
+  auto bail = [&](int code) {
+    gf_destroy(m);
+    return code;
+  };
+  if (cudaGetDevice(&m->dev) != cudaSuccess) return bail(fail(GF_ECUDA, "no CUDA device"));
+  cudaDeviceGetAttribute(&m->sms, cudaDevAttrMultiProcessorCount, m->dev);
+  int major = 0, minor = 0;
+  cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, m->dev);
+  cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, m->dev);
+  if (major != 10) return bail(fail(GF_ENOTIMPL, "needs a Blackwell (sm_10x) GPU, found sm_%d%d", major, minor));
+  m->L = c.layers;
+  m->d = c.d_model;
+  m->nq = c.n_q;
+  m->nkv = c.n_kv;
+  m->hd = c.head_dim;
+  m->ffn = c.ffn;
+  m->ffn_pad = (c.ffn + 63) / 64 * 64;
+  m->vocab = c.vocab;
+  m->q_dim = c.n_q * c.head_dim;
+  m->qkv_dim = (c.n_q + 2 * c.n_kv) * c.head_dim;
+  m->B_max = c.max_batch;
+  m->T_max = c.max_prefill_tokens;
+  m->max_pages = (c.max_seq + 63) / 64;
+  m->num_pages = c.kv_pages > 0 ? c.kv_pages : (int64_t)c.max_batch * m->max_pages;
+  if ((int64_t)m->L * m->num_pages * m->nkv * 64 >= ((int64_t)1 << 31))
+    return bail(fail(GF_ENOTIMPL, "KV pool too large for 32-bit TMA row coordinates"));
+  m->dec_max_splits = (c.max_seq + m->dec_chunk - 1) / m->dec_chunk;
+
+  // ---- weights
+  const int d = m->d, hd = m->hd;
+  m->layers.resize(m->L);
+  for (int l = 0; l < m->L && rc == GF_OK; ++l) {
+    gf_model::Layer& W = m->layers[l];
+    rc = dalloc(m, &W.qkv, (size_t)m->qkv_dim * d);
+    if (!rc) rc = dalloc(m, &W.o, (size_t)d * m->q_dim);
+    if (!rc) rc = dalloc(m, &W.gu, (size_t)2 * m->ffn_pad * d);
+    if (!rc) rc = dalloc(m, &W.down, (size_t)d * m->ffn_pad);
+    if (!rc) rc = dalloc(m, &W.attn_norm, d);
+    if (!rc) rc = dalloc(m, &W.ffn_norm, d);
+  }
+  if (!rc) rc = dalloc(m, &m->embed, (size_t)m->vocab * d);
+  if (!rc) rc = dalloc(m, &m->head, (size_t)m->vocab * d);
+  if (!rc) rc = dalloc(m, &m->final_norm, d);
+  // ---- KV pool, tables
+  const size_t cache_elems = (size_t)m->L * m->num_pages * m->nkv * 64 * hd;
+  if (!rc) rc = dalloc(m, &m->k_cache, cache_elems);
+  if (!rc) rc = dalloc(m, &m->v_cache, cache_elems);
+  if (!rc) rc = dalloc(m, &m->bt, (size_t)m->B_max * m->max_pages);
+  if (!rc) rc = dalloc(m, &m->seq_len, m->B_max);
+  if (!rc) rc = dalloc(m, &m->rope_cs, (size_t)c.max_seq * (hd / 2));
+  // ---- activations
+  const size_t T = (size_t)m->T_max;
+  if (!rc) rc = dalloc(m, &m->resid, T * d);
+  if (!rc) rc = dalloc(m, &m->xn, T * d);
+  if (!rc) rc = dalloc(m, &m->qkv, T * m->qkv_dim);
+  if (!rc) rc = dalloc(m, &m->q, T * m->q_dim);
+  if (!rc) rc = dalloc(m, &m->attn, T * m->q_dim);
+  if (!rc) rc = dalloc(m, &m->act, T * m->ffn_pad);
+  if (!rc) rc = dalloc(m, &m->prompt_ids, T);
+  if (!rc) rc = dalloc(m, &m->in_ids, T);
+  const size_t Bm = (size_t)m->B_max;
+  if (!rc) rc = dalloc(m, &m->dres, Bm * d);
+  if (!rc) rc = dalloc(m, &m->dxn, Bm * d);
+  if (!rc) rc = dalloc(m, &m->dqkv, Bm * m->qkv_dim);
+  if (!rc) rc = dalloc(m, &m->dq, Bm * m->q_dim);
+  if (!rc) rc = dalloc(m, &m->dattn, Bm * m->q_dim);
+  if (!rc) rc = dalloc(m, &m->dact, Bm * m->ffn_pad);
+  if (!rc) rc = dalloc(m, &m->part_o, Bm * m->nkv * m->dec_max_splits * 16 * hd);
+  if (!rc) rc = dalloc(m, &m->part_ml, Bm * m->nkv * m->dec_max_splits * 16 * 2);
+  if (!rc) rc = dalloc(m, &m->logits, Bm * m->vocab);
+  if (!rc) rc = dalloc(m, &m->last_idx, Bm);
+  if (!rc) rc = dalloc(m, &m->next, Bm);
+  if (!rc) rc = dalloc(m, &m->handles, Bm);
+  m->call_ints = 2 * Bm + 8 + 2 * (size_t)(T / 128 + Bm + 8);
+  if (!rc) rc = dalloc(m, &m->call, m->call_ints);
+  if (!rc) rc = dalloc(m, &m->fcall, 3 * Bm + 8);
+  if (!rc) rc = dalloc(m, &m->out_small, Bm * 12);
+  if (!rc) rc = dalloc(m, &m->err, 1);
+  if (rc) return bail(rc);
+
+  // ---- pack weights
+  auto cp = [&](void* dst, const void* src, size_t bytes) {
+    return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, s);
+  };
+  cudaError_t e = cudaSuccess;
+  const size_t qb = (size_t)m->q_dim * d * 2, kb = (size_t)m->nkv * hd * d * 2;
+  for (int l = 0; l < m->L && e == cudaSuccess; ++l) {
+    gf_model::Layer& W = m->layers[l];
+    if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->w_gate[l] || !w->w_up[l] || !w->w_down[l] ||
+        !w->attn_norm[l] || !w->ffn_norm[l])
+      return bail(fail(GF_EINVAL, "null weight pointer in layer %d", l));
+    e = cp(W.qkv, w->wq[l], qb);
+    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(W.qkv) + qb, w->wk[l], kb);
+    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(W.qkv) + qb + kb, w->wv[l], kb);
+    if (e == cudaSuccess) e = cp(W.o, w->wo[l], (size_t)d * m->q_dim * 2);
+    if (e == cudaSuccess)
+      e = gf::launch_pack_gate_up(reinterpret_cast<const bf16*>(w->w_gate[l]),
+                                  reinterpret_cast<const bf16*>(w->w_up[l]), m->ffn, m->ffn_pad, d, W.gu, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(W.down, 0, (size_t)d * m->ffn_pad * 2, s);
+    if (e == cudaSuccess)
+      e = cudaMemcpy2DAsync(W.down, (size_t)m->ffn_pad * 2, w->w_down[l], (size_t)m->ffn * 2, (size_t)m->ffn * 2, d,
+                            cudaMemcpyDeviceToDevice, s);
+    if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->attn_norm[l]), d, W.attn_norm, s);
+    if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->ffn_norm[l]), d, W.ffn_norm, s);
+  }
+  if (e == cudaSuccess) e = cp(m->embed, w->embed, (size_t)m->vocab * d * 2);
+  if (e == cudaSuccess) e = cp(m->head, w->lm_head, (size_t)m->vocab * d * 2);
+  if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->final_norm), d, m->final_norm, s);
+  if (e == cudaSuccess) e = gf::launch_rope_table(c.rope_theta, hd, c.max_seq, m->rope_cs, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(m->dqkv, 0, Bm * m->qkv_dim * sizeof(float), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(m->err, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(m->seq_len, 0, Bm * sizeof(int32_t), s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return bail(fail(GF_ECUDA, "weight packing failed: %s", cudaGetErrorString(e)));
+
+  // ---- host state
+  m->h_bt.assign((size_t)m->B_max * m->max_pages, -1);
+  m->h_len.assign(m->B_max, 0);
+  m->live.assign(m->B_max, 0);
+  m->free_pages.reserve(m->num_pages);
+  for (int64_t p = m->num_pages - 1; p >= 0; --p) m->free_pages.push_back((int32_t)p);
+  for (int sl = m->B_max - 1; sl >= 0; --sl) m->free_slots.push_back(sl);
+  const uint64_t rows = (uint64_t)m->L * m->num_pages * m->nkv * 64;
+  if ((rc = make_map(&m->tm_k, m->k_cache, hd, rows, hd * 2, 64, 64))) return bail(rc);
+  if ((rc = make_map(&m->tm_v, m->v_cache, hd, rows, hd * 2, 64, 64))) return bail(rc);
+  if ((rc = upload_block_table(m, s))) return bail(rc);
+  if (cudaStreamSynchronize(s) != cudaSuccess) return bail(fail(GF_ECUDA, "create: sync failed"));
+  *out = m;
+  return GF_OK;
+}
+
+int gf_prefill(gf_model* m, int32_t B, const int32_t* ids, const int32_t* offsets, int32_t* seq_handles,
+               float* last_logits, int32_t* next_ids, void* stream) {
+  if (!m || !seq_handles) return fail(GF_EINVAL, "null argument");
+  return prefill_impl(m, B, ids, offsets, 0, seq_handles, last_logits, next_ids,
+                      reinterpret_cast<cudaStream_t>(stream));
+}
+
+int gf_decode_step(gf_model* m, int32_t B, const int32_t* seq_handles, const int32_t* ids, float* logits,
+                   int32_t* next_ids, void* stream) {
+  if (!m || !seq_handles || !ids) return fail(GF_EINVAL, "null argument");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  TRY(prepare_decode(m, B, seq_handles, s));
+  TRY(upload(m->staging, m->handles, seq_handles, (size_t)B * sizeof(int32_t), s));
+  return decode_impl(m, B, seq_handles, ids, logits, next_ids, nullptr, 0, s);
+}
+
+int gf_release(gf_model* m, int32_t B, const int32_t* seq_handles) {
+  if (!m || (B > 0 && !seq_handles)) return fail(GF_EINVAL, "null argument");
+  for (int b = 0; b < B; ++b) {
+    const int h = seq_handles[b];
+    if (h < 0 || h >= m->B_max || !m->live[h]) return fail(GF_EINVAL, "handle %d is not live", h);
+  }
+  for (int b = 0; b < B; ++b) release_slot(m, seq_handles[b]);
+  return GF_OK;
+}
+
+int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdict_ids, int32_t K, float tau,
+               float* p, float* conf, int32_t* verdict_arg, uint8_t* defer, void* stream) {
+  if (B < 0 || !logits || !verdict_ids || !p || !conf || !verdict_arg || !defer)
+    return fail(GF_EINVAL, "null argument");
+  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
+  if (!(tau >= 0.f && tau <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
+  for (int k = 0; k < K; ++k)
+    if (verdict_ids[k] < 0 || verdict_ids[k] >= ld) return fail(GF_EINVAL, "verdict id %d outside the row", verdict_ids[k]);
+  CU(gf::launch_verdict(logits, ld, B, verdict_ids, K, tau, p, conf, verdict_arg, defer,
+                        reinterpret_cast<cudaStream_t>(stream)));
+  return GF_OK;
+}
+
+int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                      const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                      const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                      int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, float* final_logits, void* stream) {
+  if (!m || !inc_offsets || !cand_offsets || !verdict_ids || !p || !conf || !verdict_arg || !defer)
+    return fail(GF_EINVAL, "null argument");
+  if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
+  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
+  if (!(tau >= 0.f && tau <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
+  if (n_decode < 0) return fail(GF_EINVAL, "n_decode < 0");
+  for (int k = 0; k < K; ++k)
+    if (verdict_ids[k] < 0 || verdict_ids[k] >= m->vocab) return fail(GF_EINVAL, "verdict id %d >= vocab", verdict_ids[k]);
+  if (inc_offsets[0] != 0 || cand_offsets[0] != 0) return fail(GF_EINVAL, "offsets must start at 0");
+  std::vector<int32_t> poff(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int ni = inc_offsets[b + 1] - inc_offsets[b], nc = cand_offsets[b + 1] - cand_offsets[b];
+    if (ni < 0 || nc < 0 || ni + nc < 1) return fail(GF_EINVAL, "item %d: bad lengths %d + %d", b, ni, nc);
+    if ((ni > 0 && !inc_ids) || (nc > 0 && !cand_ids)) return fail(GF_EINVAL, "null ids");
+    poff[b + 1] = poff[b] + ni + nc;
+  }
+  if (poff[B] > m->T_max) return fail(GF_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int32_t> desc;
+  desc.insert(desc.end(), inc_offsets, inc_offsets + B + 1);
+  desc.insert(desc.end(), cand_offsets, cand_offsets + B + 1);
+  desc.insert(desc.end(), poff.begin(), poff.end());
+  TRY(upload(m->staging, m->fcall, desc.data(), desc.size() * sizeof(int32_t), s));
+  CU(gf::launch_build_prompts(inc_ids, m->fcall, cand_ids, m->fcall + B + 1, m->fcall + 2 * (B + 1), B, poff[B],
+                              m->prompt_ids, s));
+  m->launches++;
+  std::vector<int32_t> h(B);
+  float* lg = (n_decode == 0 && final_logits) ? final_logits : m->logits;
+  // tokens[b, s] is the input of decode step s: the arg max of the logits before it
+  TRY(prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), lg, m->next, s,
+                   (tokens && n_decode > 0) ? tokens : nullptr, n_decode));
+  int rc = upload(m->staging, m->handles, h.data(), (size_t)B * sizeof(int32_t), s);
+  for (int step = 0; step < n_decode && rc == GF_OK; ++step) {
+    float* dst = (step == n_decode - 1 && final_logits) ? final_logits : m->logits;
+    lg = dst;
+    int32_t* col = (tokens && step + 1 < n_decode) ? tokens + step + 1 : nullptr;
+    rc = decode_impl(m, B, h.data(), m->next, dst, m->next, col, n_decode, s);
+  }
+  if (rc == GF_OK) {
+    const cudaError_t e = gf::launch_verdict(lg, m->vocab, B, verdict_ids, K, tau, p, conf, verdict_arg, defer, s);
+    if (e != cudaSuccess) rc = fail(GF_ECUDA, "verdict launch: %s", cudaGetErrorString(e));
+    m->launches++;
+  }
+  for (int b = 0; b < B; ++b) release_slot(m, h[b]);
+  return rc;
+}
+
+int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                           const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                           const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                           int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, void* stream) {
+  if (!m || !inc_offsets || !cand_offsets || !p || !conf || !verdict_arg || !defer)
+    return fail(GF_EINVAL, "null argument");
+  if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
+  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int64_t ni = inc_offsets[B], nc = cand_offsets[B];
+  if (ni < 0 || nc < 0 || ni + nc > m->T_max) return fail(GF_ECAPACITY, "ids exceed max_prefill_tokens");
+  TRY(upload(m->staging, m->in_ids, inc_ids, (size_t)ni * sizeof(int32_t), s));
+  TRY(upload(m->staging, m->in_ids + ni, cand_ids, (size_t)nc * sizeof(int32_t), s));
+  // outputs on the device: p [B*K] | conf [B] | arg [B] | defer [B]  (within out_small, B_max*12 floats)
+  float* dp = m->out_small;
+  float* dconf = dp + (size_t)B * 8;
+  int32_t* darg = reinterpret_cast<int32_t*>(dconf + B);
+  uint8_t* ddef = reinterpret_cast<uint8_t*>(darg + B);
+  // the generated tokens are staged on the device right after the prompt ids
+  int32_t* dtok = nullptr;
+  if (tokens && n_decode > 0) {
+    if (ni + nc + (int64_t)B * n_decode > m->T_max) return fail(GF_ECAPACITY, "tokens output exceeds staging");
+    dtok = m->in_ids + ni + nc;
+  }
+  TRY(gf_forecast_batch(m, B, m->in_ids, inc_offsets, m->in_ids + ni, cand_offsets, n_decode, verdict_ids, K, tau,
+                        dp, dconf, darg, ddef, dtok, nullptr, stream));
+  const size_t bytes = (size_t)B * 12 * sizeof(float) + (dtok ? (size_t)B * n_decode * sizeof(int32_t) : 0);
+  if (m->host_out_cap < bytes) {
+    if (m->host_out) cudaFreeHost(m->host_out);
+    m->host_out = nullptr;
+    m->host_out_cap = 0;
+    if (cudaHostAlloc(&m->host_out, bytes, cudaHostAllocDefault) != cudaSuccess) return fail(GF_ENOMEM, "pinned out");
+    m->host_out_cap = bytes;
+  }
+  char* ho = reinterpret_cast<char*>(m->host_out);
+  CU(cudaMemcpyAsync(ho, m->out_small, (size_t)B * 12 * sizeof(float), cudaMemcpyDeviceToHost, s));
+  if (dtok)
+    CU(cudaMemcpyAsync(ho + (size_t)B * 12 * sizeof(float), dtok, (size_t)B * n_decode * sizeof(int32_t),
+                       cudaMemcpyDeviceToHost, s));
+  CU(cudaStreamSynchronize(s));
+  const float* hp = reinterpret_cast<const float*>(ho);
+  memcpy(p, hp, (size_t)B * K * sizeof(float));
+  memcpy(conf, hp + (size_t)B * 8, (size_t)B * sizeof(float));
+  memcpy(verdict_arg, hp + (size_t)B * 9, (size_t)B * sizeof(int32_t));
+  memcpy(defer, hp + (size_t)B * 10, (size_t)B);
+  if (dtok) memcpy(tokens, ho + (size_t)B * 12 * sizeof(float), (size_t)B * n_decode * sizeof(int32_t));
+  return GF_OK;
+}
+
+static int* g_gemm_err = nullptr;
+
+int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
+                 int32_t mode, int32_t bn, int32_t splits, void* stream) {
+  if (!A || !W || !out || M < 0 || N < 1 || K < 64) return fail(GF_EINVAL, "bad GEMM arguments");
+  if (K % 64 || N % 32) return fail(GF_EINVAL, "GEMM needs K %% 64 == 0 and N %% 32 == 0");
+  if (mode < GF_GEMM_STORE_F32 || mode > GF_GEMM_SWIGLU) return fail(GF_EINVAL, "bad GEMM mode");
+  if (mode == GF_GEMM_SWIGLU && N % 128) return fail(GF_EINVAL, "SwiGLU GEMM needs N %% 128 == 0");
+  if (bn != 0 && bn != 64 && bn != 128 && bn != 256) return fail(GF_EINVAL, "bn must be 0, 64, 128 or 256");
+  if (mode == GF_GEMM_SWIGLU && bn == 64) return fail(GF_EINVAL, "SwiGLU GEMM needs bn >= 128");
+  if (splits > 1 && mode != GF_GEMM_ATOMIC_F32) return fail(GF_EINVAL, "split-K needs the atomic mode");
+  if (ldo < (mode == GF_GEMM_SWIGLU ? N / 2 : N)) return fail(GF_EINVAL, "ldo too small");
+  if (M == 0) return GF_OK;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (!g_gemm_err) {
+    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
+    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
+  }
+  int dev = 0, sms = 0;
+  CU(cudaGetDevice(&dev));
+  CU(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  gf_model fake;
+  fake.sms = sms;
+  int pbn, psplits;
+  plan_gemm(&fake, M, N, K, mode, &pbn, &psplits);
+  if (bn == 0) bn = pbn;
+  if (splits <= 0) splits = psplits;
+  CUtensorMap ta, tb;
+  TRY(make_map(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, 128));
+  TRY(make_map(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, (uint32_t)bn));
+  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s));
+  return GF_OK;
+}
+
+int gf_gemm_status(void* stream) {
+  CU(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
+  if (!g_gemm_err) return GF_OK;
+  int h = 0;
+  CU(cudaMemcpy(&h, g_gemm_err, sizeof(int), cudaMemcpyDeviceToHost));
+  CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
+  if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a GEMM wait timed out");
+  return GF_OK;
+}
+
+int gf_profile_enable(gf_model* m, uint32_t mask) {
+  if (!m) return fail(GF_EINVAL, "null model");
+  m->prof_mask = mask;
+  return GF_OK;
+}
+
+int gf_profile_read(gf_model* m, int32_t kind, int64_t* launches, double* ms, double* flops, double* bytes) {
+  if (!m || kind < 0 || kind >= GF_PROF_KINDS) return fail(GF_EINVAL, "bad profile request");
+  CU(cudaDeviceSynchronize());
+  int64_t n = 0;
+  double t = 0, f = 0, by = 0;
+  std::vector<gf_model::ProfRec> keep;
+  for (auto& r : m->prof) {
+    if (r.kind != kind) {
+      keep.push_back(r);
+      continue;
+    }
+    float e = 0.f;
+    CU(cudaEventElapsedTime(&e, r.a, r.b));
+    ++n;
+    t += e;
+    f += r.flops;
+    by += r.bytes;
+    m->ev_pool.push_back(r.a);
+    m->ev_pool.push_back(r.b);
+  }
+  m->prof.swap(keep);
+  if (launches) *launches = n;
+  if (ms) *ms = t;
+  if (flops) *flops = f;
+  if (bytes) *bytes = by;
+  return GF_OK;
+}
+
+int gf_debug_capture(gf_model* m, int32_t layer, int32_t item, float* dst, int64_t cap_rows) {
+  if (!m || !dst || layer < 0 || layer > m->L || item < 0 || item >= m->B_max || cap_rows < 1)
+    return fail(GF_EINVAL, "bad capture request");
+  if (m->caps.size() >= 8) return fail(GF_ECAPACITY, "too many captures armed");
+  m->caps.push_back({layer, item, dst, cap_rows});
+  return GF_OK;
+}
+
+int gf_debug_read_kv(gf_model* m, int32_t layer, int32_t handle, int32_t start, int32_t n, void* k_dst,
+                     void* v_dst, void* stream) {
+  if (!m || !k_dst || !v_dst || layer < 0 || layer >= m->L || handle < 0 || handle >= m->B_max ||
+      !m->live[handle] || start < 0 || n < 0 || start + n > m->h_len[handle])
+    return fail(GF_EINVAL, "bad KV read request");
+  CU(gf::launch_read_kv(m->k_cache, m->v_cache, m->bt, m->max_pages, handle, start, n, m->nkv, m->hd,
+                        layer_row0(m, layer), reinterpret_cast<bf16*>(k_dst), reinterpret_cast<bf16*>(v_dst),
+                        reinterpret_cast<cudaStream_t>(stream)));
+  return GF_OK;
+}
+
+int gf_device_status(gf_model* m, void* stream) {
+  if (!m) return fail(GF_EINVAL, "null model");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  CU(cudaStreamSynchronize(s));
+  int h = 0;
+  CU(cudaMemcpy(&h, m->err, sizeof(int), cudaMemcpyDeviceToHost));
+  CU(cudaMemset(m->err, 0, sizeof(int)));
+  if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a device-side wait timed out");
+  if (h == 1) return fail(GF_EINVAL, "a token id outside [0, vocab) reached the device");
+  if (h != 0) return fail(GF_ECUDA, "device error word %d", h);
+  return GF_OK;
+}
+
+}  // extern "C"

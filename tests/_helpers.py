@@ -1,0 +1,75 @@
+"""Shared test helpers: synthetic weights on the device, tolerance checks."""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+
+# Final logits: |gpu - oracle| <= ATOL + RTOL * |oracle| (bf16 path vs float64 oracle).
+LOGIT_ATOL = 3e-2
+LOGIT_RTOL = 2e-2
+# Verdict probabilities: absolute.
+P_ATOL = 1e-2
+# Greedy arg max may differ when the oracle's top-2 logit gap is below this.
+ARGMAX_GAP = 3e-2
+# The defer bit may differ when the oracle's confidence is this close to tau.
+DEFER_BAND = 1e-2
+
+
+def to_device_bf16(bits: np.ndarray):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def device_weights(shape: synth.ModelShape, seed: int = 0) -> dict:
+    """The synth weights of `shape` as bf16 CUDA tensors, in the layout gf_create takes."""
+    W = {"embed": to_device_bf16(synth.embed_bf16(shape, seed)),
+         "lm_head": to_device_bf16(synth.head_bf16(shape, seed)),
+         "final_norm": to_device_bf16(synth.ones_bf16(shape.d_model))}
+    for k in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down"):
+        W[k] = []
+    for l in range(shape.layers):
+        lw = synth.layer_weights_bf16(shape, l, seed)
+        for k, v in lw.items():
+            W[k].append(to_device_bf16(v))
+        W["attn_norm"].append(to_device_bf16(synth.ones_bf16(shape.d_model)))
+        W["ffn_norm"].append(to_device_bf16(synth.ones_bf16(shape.d_model)))
+    return W
+
+
+def make_model(shape, max_batch, max_seq, max_prefill_tokens, seed=0, kv_pages=0):
+    import paper_2605_31464_gb300 as gf
+    W = device_weights(shape, seed)
+    m = gf.Model(shape, W, max_batch=max_batch, max_seq=max_seq, max_prefill_tokens=max_prefill_tokens,
+                 kv_pages=kv_pages)
+    del W
+    return m
+
+
+def check_logits(gpu: np.ndarray, ref: np.ndarray, what: str = "logits"):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    err = np.abs(gpu - ref)
+    bound = LOGIT_ATOL + LOGIT_RTOL * np.abs(ref)
+    bad = err > bound
+    assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} outside tolerance; max err {err.max():.4g}, "
+                           f"worst at {np.unravel_index(np.argmax(err - bound), err.shape)}")
+    return float(err.max())
+
+
+def greedy_agrees(gpu_tok: int, ref_logits: np.ndarray) -> bool:
+    """GPU arg max equals the oracle's, or the oracle's top-2 gap is within the tie band."""
+    order = np.argsort(-ref_logits, kind="stable")
+    top1 = int(order[0])
+    if gpu_tok == top1:
+        return True
+    return ref_logits[top1] - ref_logits[gpu_tok] < ARGMAX_GAP
+
+
+def check_verdict(gpu_p, gpu_conf, gpu_arg, gpu_defer, ref_p, ref_conf, ref_arg, ref_defer, tau):
+    np.testing.assert_allclose(np.asarray(gpu_p, dtype=np.float64), ref_p, atol=P_ATOL, rtol=0)
+    np.testing.assert_allclose(float(gpu_conf), ref_conf, atol=P_ATOL, rtol=0)
+    srt = np.sort(ref_p)[::-1]
+    if len(srt) < 2 or srt[0] - srt[1] >= 2e-2:
+        assert int(gpu_arg) == int(ref_arg)
+    if abs(ref_conf - tau) >= DEFER_BAND:
+        assert int(gpu_defer) == int(ref_defer)
