@@ -1,0 +1,353 @@
+#!/usr/bin/env python
+"""Throughput of the surrogate forecaster's hot path on GB300.
+
+One step = one call of gf_forecast_batch on a batch of candidates: prefill of
+every prompt, n_decode greedy decode steps (the reasoning trace), then the
+verdict softmax, confidence and defer mask at tau (Sec. 2.1).  The default
+workload is the 7B-class prefill-bound configuration (28 layers, d 3584,
+GQA 28/4 x 128, SwiGLU 18944, vocab 152064; 32 prompts of 6144 Zipf(1.1)
+ids, 256 decode steps, tau 0.8).  Weights and ids are seeded synthetic
+(``synth``); the weights (14 GB) exceed L2, so no flush is needed.
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the float64 CPU
+oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+# DRAM bytes per launch of the dominant kernel, from an ncu capture of the
+# same kernel build (profiles/), or None when no capture of this build exists.
+NCU_TRAFFIC = {}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="7b_prefill", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0, help="override the batch (testing only)")
+    return ap.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sus=p["bf16_tflops_sustained"], src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+def workload_config(w: synth.Workload, world: int) -> dict:
+    m = w.model
+    return {"workload": w.name,
+            "model": f"{m.layers}L d{m.d_model} GQA {m.n_q}/{m.n_kv}x{m.head_dim} ffn {m.ffn} vocab {m.vocab}",
+            "batch_per_gpu": w.batch, "global_batch": w.batch * world,
+            "prompt_len": w.prompt_len if w.ragged is None else f"U[{w.ragged[0]},{w.ragged[1]}]",
+            "incumbent_len": w.inc_len, "ids": w.id_dist, "n_decode": w.n_decode, "tau": w.tau,
+            "verdict_ids": list(w.verdict_ids), "parallelism": f"replicas x{world}" if world > 1 else "1 GPU",
+            "l2": "inputs larger than L2 (bf16 weights stream every step)"}
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(prefix="clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        self.proc.wait()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle sample
+def cpu_oracle_sample(w: synth.Workload):
+    """Time the float64 oracle on one item and one layer at full prompt length,
+    plus one decode-step layer at that context and the LM head on one row;
+    extrapolate to a whole forecast (all layers, all decode steps)."""
+    import oracle
+    m = w.model
+    ids, off = synth.packed_prompts(w, items=[0])
+    P = int(off[1])
+    W = oracle.Weights(m, cache_layers=False)
+    lw = W.layer(0)
+    x = W.embed_rows(ids)
+    t0 = time.perf_counter()
+    y, k, v = oracle.layer_forward(x, lw, m, np.arange(P))
+    t_layer = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    oracle.layer_forward(y[-1:], lw, m, np.array([P]), k, v)
+    t_dec_layer = time.perf_counter() - t0
+    W.head()
+    t0 = time.perf_counter()
+    oracle.lm_head(y[-1:], W)
+    t_head = time.perf_counter() - t0
+    per_forecast = m.layers * t_layer + t_head + w.n_decode * (m.layers * t_dec_layer + t_head)
+    cores = len(os.sched_getaffinity(0))
+    sample = (f"1 item, layer 1 of {m.layers} at prompt {P} ({t_layer:.2f} s) + 1 decode-step layer at context {P} "
+              f"({t_dec_layer * 1e3:.1f} ms) + LM head ({t_head * 1e3:.1f} ms); extrapolated x{m.layers} layers, "
+              f"x{w.n_decode} decode steps")
+    return 1.0 / per_forecast, cores, sample, t_layer + t_dec_layer + t_head
+
+
+# ----------------------------------------------------------------------------- reference arm
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    w = synth.workload(args.workload)
+    cfg = workload_config(w, 1)
+    vals, secs = [], []
+    for i in range(args.warmup + args.steps):
+        v, cores, sample, sec = cpu_oracle_sample(w)
+        if i >= args.warmup:
+            vals.append(v)
+            secs.append(sec)
+    value = float(np.mean(vals))
+    line = {"impl": "reference", "metric": "forecasts/s", "value": value, "unit": "forecasts/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * float(np.mean(secs)),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": cfg,
+            "cpu_baseline": {"value": value, "unit": "forecasts/s", "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "forecasts/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ----------------------------------------------------------------------------- our arm
+def device_weights(m: synth.ModelShape):
+    import torch
+
+    def dev(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+    W = {"embed": dev(synth.embed_bf16(m)), "lm_head": dev(synth.head_bf16(m)),
+         "final_norm": dev(synth.ones_bf16(m.d_model))}
+    for k in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down"):
+        W[k] = []
+    for l in range(m.layers):
+        for k, v in synth.layer_weights_bf16(m, l).items():
+            W[k].append(dev(v))
+        W["attn_norm"].append(dev(synth.ones_bf16(m.d_model)))
+        W["ffn_norm"].append(dev(synth.ones_bf16(m.d_model)))
+    return W
+
+
+def run_ours(args):
+    import torch
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    from paper_2605_31464_gb300 import _build
+    if rank == 0:
+        _build.build()
+    if world > 1:
+        torch.distributed.barrier()
+    import paper_2605_31464_gb300 as gf
+
+    base = synth.workload(args.workload)
+    B = args.batch or base.batch
+    # weak scaling: every rank forecasts its own B candidates (items rank*B ... rank*B+B-1)
+    w_all = synth.workload(args.workload, batch=B * world)
+    items = list(range(rank * B, rank * B + B))
+    w = synth.workload(args.workload, batch=B)
+    m = w.model
+    inc, io, cand, co = synth.prompts(w_all, items=items)
+    lens = np.diff(io) + np.diff(co)
+    max_len = int(lens.max())
+
+    W = device_weights(m)
+    model = gf.Model(m, W, max_batch=B, max_seq=max_len + w.n_decode, max_prefill_tokens=int(lens.sum()) +
+                     B * w.n_decode + 64)
+    del W
+    torch.cuda.empty_cache()
+    inc_d = torch.from_numpy(inc).cuda()
+    cand_d = torch.from_numpy(cand).cuda()
+
+    def step():
+        return model.forecast_batch(inc_d, io, cand_d, co, w.n_decode, w.verdict_ids, w.tau, want_tokens=False)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    model.status()
+    pk = peaks()
+    model.profile(1 << gf.GF_PROF_PREFILL_GEMM)
+    for k in range(4):
+        model.profile_read(k)
+    clocks = ClockSampler(local)
+    launches0 = model.launch_count()
+    stream = torch.cuda.current_stream()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        out = step()
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    clk = clocks.stop()
+    launches = model.launch_count() - launches0
+    ms = ev0.elapsed_time(ev1)
+    prof = model.profile_read(gf.GF_PROF_PREFILL_GEMM)
+    model.profile(0)
+    model.status()
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    defer_frac = float(out["defer"].float().mean().item())
+    value = B * world * args.steps / (ms / 1e3)
+
+    # ---- end to end through the host-buffer entry point (copies inside the timed region)
+    model.forecast_batch_host(inc, io, cand, co, w.n_decode, w.verdict_ids, w.tau, want_tokens=True)
+    if world > 1:
+        torch.distributed.barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        model.forecast_batch_host(inc, io, cand, co, w.n_decode, w.verdict_ids, w.tau, want_tokens=True)
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    K = len(w.verdict_ids)
+    h2d = int(inc.nbytes + cand.nbytes + io.nbytes + co.nbytes)
+    d2h = int(B * (K * 4 + 4 + 4 + 1) + B * w.n_decode * 4)
+
+    # ---- prefill / decode split (outside the timed region)
+    ids_p, off_p = [], [0]
+    for i in range(B):
+        seq = np.concatenate([inc[io[i]:io[i + 1]], cand[co[i]:co[i + 1]]])
+        ids_p.append(seq)
+        off_p.append(off_p[-1] + len(seq))
+    ids_d = torch.from_numpy(np.concatenate(ids_p).astype(np.int32)).cuda()
+    model.profile((1 << gf.GF_PROF_DECODE_GEMM) | (1 << gf.GF_PROF_DECODE_ATTN) | (1 << gf.GF_PROF_PREFILL_ATTN))
+    e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+    e0.record(stream)
+    h, _, nxt = model.prefill(ids_d, off_p, want_logits=False)
+    e1.record(stream)
+    n_dec_probe = min(32, w.n_decode)
+    for _ in range(n_dec_probe):
+        _, nxt = model.decode_step(h, nxt, want_logits=False)
+    e2.record(stream)
+    torch.cuda.synchronize()
+    model.release(h)
+    prefill_ms = e0.elapsed_time(e1)
+    decode_ms = e1.elapsed_time(e2) / max(n_dec_probe, 1)
+    dgemm = model.profile_read(gf.GF_PROF_DECODE_GEMM)
+    dattn = model.profile_read(gf.GF_PROF_DECODE_ATTN)
+    pattn = model.profile_read(gf.GF_PROF_PREFILL_ATTN)
+    model.profile(0)
+
+    if rank != 0:
+        model.close()
+        return 0
+    achieved = prof["flops"] / (prof["ms"] / 1e3) / 1e12 if prof["ms"] > 0 else 0.0
+    traffic = NCU_TRAFFIC.get(args.workload)
+    roofline = {"bound": "tensor", "kernel": "gemm_tc_kernel (prefill launches: QKV, O, gate/up+SwiGLU, down, LM head)",
+                "achieved": achieved, "peak": pk["bf16_sus"], "unit": "TFLOP/s",
+                "frac": achieved / pk["bf16_sus"], "traffic": traffic,
+                "peak_note": f"bf16 sustained, {pk['src']} (MEASURED_PEAKS.json)",
+                "launches": prof["launches"], "avg_launch_ms": prof["ms"] / max(prof["launches"], 1),
+                "algorithmic_tflop_per_launch": prof["flops"] / max(prof["launches"], 1) / 1e12}
+    cfg = workload_config(w, world)
+    line = {"metric": "forecasts/s", "value": value, "unit": "forecasts/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic", "config": cfg, "roofline": roofline,
+            "e2e": {"value": B * world * args.steps / e2e_s, "unit": "forecasts/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": int(launches), "clocks": clk,
+            "prefill_tok_per_s": float(lens.sum()) / (prefill_ms / 1e3),
+            "decode_tok_per_s": B / (decode_ms / 1e3),
+            "prefill_ms": prefill_ms, "decode_ms_per_step": decode_ms,
+            "defer_fraction": defer_frac,
+            "decode_roofline": {
+                "gemm_GBps": dgemm["bytes"] / (dgemm["ms"] / 1e3) / 1e9 if dgemm["ms"] else None,
+                "attn_GBps": dattn["bytes"] / (dattn["ms"] / 1e3) / 1e9 if dattn["ms"] else None,
+                "gemm_ms_per_step": dgemm["ms"] / max(n_dec_probe, 1),
+                "attn_ms_per_step": dattn["ms"] / max(n_dec_probe, 1),
+                "peak_GBps": pk["hbm"], "peak_note": f"HBM copy, {pk['src']}"},
+            "prefill_attention": {"TFLOPs": pattn["flops"] / (pattn["ms"] / 1e3) / 1e12 if pattn["ms"] else None,
+                                  "ms": pattn["ms"]}}
+    if world == 1 and not args.no_cpu_baseline:
+        v, cores, sample, _ = cpu_oracle_sample(w)
+        line["cpu_baseline"] = {"value": v, "unit": "forecasts/s", "cores": cores, "kind": "oracle", "sample": sample}
+    print(json.dumps(line), flush=True)
+    model.close()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())
