@@ -180,8 +180,31 @@ enum { GF_GEMM_STORE_F32 = 0, GF_GEMM_ADD_F32 = 1, GF_GEMM_ATOMIC_F32 = 2, GF_GE
        GF_GEMM_SWIGLU = 4 };
 int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
                  int32_t mode, int32_t bn, int32_t splits, void* stream);
-/* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16 launch gave up waiting. */
+/* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16 or gf_decode_attention
+ * launch gave up waiting. */
 int gf_gemm_status(void* stream);
+
+/* Decode attention over a paged KV cache, the step a decode token spends on
+ * its context (one query token per sequence, grouped-query heads):
+ *   out[b, h, :] = sum_j softmax_j(q[b,h,:] . k_j / sqrt(hd)) v_j  over the
+ *   ctx_len[b] cached positions j of sequence b, kv head h / (n_q / n_kv).
+ *   q            device bf16 [B, n_q*hd], already rotated
+ *   k_cache, v_cache device bf16 [num_pages][n_kv][64][hd] (64-token pages)
+ *   block_table  device int32 [B][max_pages]: page of block j of sequence b
+ *   ctx_len      device int32 [B], 1 <= ctx_len[b] <= max_ctx (a larger
+ *                value is clamped to max_ctx; 0 gives a zero output row)
+ *   max_ctx      host bound on ctx_len, <= 64*max_pages (sizes the grid)
+ *   out          device bf16 [B, n_q*hd]
+ *   workspace    device scratch for the per-chunk partial results, at least
+ *                gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx) bytes,
+ *                owned by the caller and free for reuse once the call's work
+ *                on `stream` has completed.
+ * head_dim 64 or 128, n_q / n_kv <= 16.  Enqueued on `stream`. */
+size_t gf_decode_attention_workspace(int32_t B, int32_t n_kv, int32_t head_dim, int32_t max_ctx);
+int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
+                        const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len, int32_t max_ctx,
+                        int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out, void* workspace,
+                        size_t workspace_bytes, void* stream);
 
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes whose launches can be bracketed by CUDA events (on the

@@ -45,7 +45,7 @@ class gf_weights(ctypes.Structure):
 EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_release", "gf_forecast_batch",
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
-           "gf_profile_read"]
+           "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN = range(4)
@@ -79,6 +79,9 @@ def load(path: str = LIB_PATH):
         "gf_last_error": ([], ctypes.c_char_p),
         "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _p], ctypes.c_int),
         "gf_gemm_status": ([_p], ctypes.c_int),
+        "gf_decode_attention_workspace": ([_c_i32, _c_i32, _c_i32, _c_i32], ctypes.c_size_t),
+        "gf_decode_attention": ([_p, _p, _p, _c_i64, _p, _c_i32, _p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _p, _p,
+                                 ctypes.c_size_t, _p], ctypes.c_int),
         "gf_profile_enable": ([_p, ctypes.c_uint32], ctypes.c_int),
         "gf_profile_read": ([_p, _c_i32, ctypes.POINTER(_c_i64), ctypes.POINTER(ctypes.c_double),
                              ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double)], ctypes.c_int),
@@ -162,6 +165,31 @@ def gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, stream):
 
 def gf_gemm_status(stream):
     _check(load().gf_gemm_status(stream))
+
+
+def gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx) -> int:
+    return int(load().gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx))
+
+
+def gf_decode_attention(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx, B, n_q, n_kv,
+                        head_dim, out, workspace, workspace_bytes, stream):
+    _check(load().gf_decode_attention(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx, B,
+                                      n_q, n_kv, head_dim, out, workspace, workspace_bytes, stream))
+
+
+def decode_attention(q, k_cache, v_cache, block_table, ctx_len, max_ctx, n_q, n_kv, stream=None):
+    """Paged decode attention on torch tensors; allocates the workspace with torch."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    B = q.shape[0]
+    hd = k_cache.shape[-1]
+    ws_bytes = gf_decode_attention_workspace(B, n_kv, hd, max_ctx)
+    ws = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
+    out = torch.empty_like(q)
+    gf_decode_attention(q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(), k_cache.shape[0],
+                        block_table.data_ptr(), block_table.shape[1], ctx_len.data_ptr(), max_ctx, B, n_q, n_kv, hd,
+                        out.data_ptr(), ws.data_ptr(), ws_bytes, s.cuda_stream)
+    return out
 
 
 def gf_profile_enable(model, mask):

@@ -37,8 +37,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int split = blockIdx.x;
   const int kvh = blockIdx.y;
   const int b = blockIdx.z;
-  const int slot = a.handles[b];
-  const int ctx = a.seq_len[slot] + 1;
+  const int slot = a.handles ? a.handles[b] : b;
+  const int ctx = min(a.seq_len[slot] + a.ctx_bias, a.max_ctx);
   const int k0 = split * a.chunk;
   if (k0 >= ctx) return;
   const int k1 = min(k0 + a.chunk, ctx);
@@ -238,8 +238,8 @@ __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
   const int h = blockIdx.x % a.n_q;
   const int G = a.n_q / a.n_kv;
   const int kvh = h / G, r = h % G;
-  const int ctx = a.seq_len[a.handles[b]] + 1;
-  const int n_splits = (ctx + a.chunk - 1) / a.chunk;
+  const int ctx = min(a.seq_len[a.handles ? a.handles[b] : b] + a.ctx_bias, a.max_ctx);
+  const int n_splits = ctx > 0 ? min((ctx + a.chunk - 1) / a.chunk, a.max_splits) : 0;
   const int64_t base = ((int64_t)b * a.n_kv + kvh) * a.max_splits;
   float M = -INFINITY;
   for (int s = 0; s < n_splits; ++s) M = fmaxf(M, a.part_ml[((base + s) * 16 + r) * 2]);

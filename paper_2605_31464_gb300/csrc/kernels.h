@@ -38,8 +38,10 @@ cudaError_t launch_attn_prefill(int hd, const CUtensorMap& tmQ, const CUtensorMa
 struct DecodeAttnArgs {
   const bf16* q;              // [B, n_q*hd], rotated queries of this step
   int64_t ldq;
-  const int32_t* handles;     // [B] slots
-  const int32_t* seq_len;     // [slots] tokens cached before this step; context = seq_len + 1
+  const int32_t* handles;     // [B] slots, or nullptr: slot = b
+  const int32_t* seq_len;     // [slots]; visible keys = min(seq_len[slot] + ctx_bias, max_ctx)
+  int ctx_bias;
+  int max_ctx;
   const int32_t* block_table;
   int max_pages;
   int n_q, n_kv;

@@ -549,6 +549,8 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     da.ldq = m->q_dim;
     da.handles = m->handles;
     da.seq_len = m->seq_len;
+    da.ctx_bias = 1;
+    da.max_ctx = m->dec_max_splits * m->dec_chunk;
     da.block_table = m->bt;
     da.max_pages = m->max_pages;
     da.n_q = m->nq;
@@ -958,11 +960,61 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
 
 int gf_gemm_status(void* stream) {
   CU(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
-  if (!g_gemm_err) return GF_OK;
+  if (!g_gemm_err) return GF_OK;  // shared by gf_gemm_bf16 and gf_decode_attention
   int h = 0;
   CU(cudaMemcpy(&h, g_gemm_err, sizeof(int), cudaMemcpyDeviceToHost));
   CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
   if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a GEMM wait timed out");
+  return GF_OK;
+}
+
+size_t gf_decode_attention_workspace(int32_t B, int32_t n_kv, int32_t head_dim, int32_t max_ctx) {
+  if (B < 1 || n_kv < 1 || head_dim < 1 || max_ctx < 1) return 0;
+  const size_t splits = (size_t)(max_ctx + 255) / 256;
+  return (size_t)B * n_kv * splits * 16 * ((size_t)head_dim + 2) * sizeof(float);
+}
+
+int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
+                        const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len, int32_t max_ctx,
+                        int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out, void* workspace,
+                        size_t workspace_bytes, void* stream) {
+  if (!q || !k_cache || !v_cache || !block_table || !ctx_len || !out || !workspace)
+    return fail(GF_EINVAL, "null argument");
+  if (B < 1 || n_q < 1 || n_kv < 1 || n_q % n_kv || n_q / n_kv > 16) return fail(GF_EINVAL, "bad head counts");
+  if (head_dim != 64 && head_dim != 128) return fail(GF_ENOTIMPL, "head_dim must be 64 or 128");
+  if (max_ctx < 1 || max_pages < 1 || max_ctx > max_pages * 64) return fail(GF_EINVAL, "max_ctx outside 1..64*max_pages");
+  if (num_pages < 1 || num_pages * n_kv * 64 >= ((int64_t)1 << 31)) return fail(GF_EINVAL, "bad page count");
+  if (workspace_bytes < gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx))
+    return fail(GF_EINVAL, "workspace smaller than gf_decode_attention_workspace()");
+  if (!g_gemm_err) {
+    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
+    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
+  }
+  CUtensorMap tk, tv;
+  const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
+  TRY(make_map(&tk, k_cache, head_dim, rows, head_dim * 2, 64, 64));
+  TRY(make_map(&tv, v_cache, head_dim, rows, head_dim * 2, 64, 64));
+  gf::DecodeAttnArgs da{};
+  da.q = reinterpret_cast<const bf16*>(q);
+  da.ldq = (int64_t)n_q * head_dim;
+  da.handles = nullptr;
+  da.seq_len = ctx_len;
+  da.ctx_bias = 0;
+  da.max_ctx = max_ctx;
+  da.block_table = block_table;
+  da.max_pages = max_pages;
+  da.n_q = n_q;
+  da.n_kv = n_kv;
+  da.layer_row0 = 0;
+  da.chunk = 256;
+  da.max_splits = (max_ctx + 255) / 256;
+  da.part_o = reinterpret_cast<float*>(workspace);
+  da.part_ml = da.part_o + (size_t)B * n_kv * da.max_splits * 16 * head_dim;
+  da.out = reinterpret_cast<bf16*>(out);
+  da.ldo = (int64_t)n_q * head_dim;
+  da.scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
+  da.err = g_gemm_err;
+  CU(gf::launch_attn_decode(head_dim, tk, tv, da, B, reinterpret_cast<cudaStream_t>(stream)));
   return GF_OK;
 }
 
