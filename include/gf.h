@@ -206,6 +206,33 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
                         int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out, void* workspace,
                         size_t workspace_bytes, void* stream);
 
+/* gf_decode_attention without any allocation.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory
+ * where they call it - for example a serving loop whose device memory is
+ * already fully reserved by another allocator (a raw cudaMalloc there can
+ * fail), or code that must not call cudaMalloc/cudaFree after start-up
+ * because those calls can synchronise the whole device and stall other
+ * streams.  Arguments and results are those of gf_decode_attention; there is
+ * no workspace argument.  Instead the per-chunk partial results live in a
+ * fixed 16 MiB device array of the library (every GPU that loads the library
+ * holds it until the process exits):
+ *   - gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx) must not
+ *     exceed 16 MiB (16777216 bytes), else GF_ECAPACITY ("exceeds scratch")
+ *     and nothing is enqueued;
+ *   - the first call on a device, with that device current, looks up the
+ *     array's device address (cudaGetSymbolAddress); make that first call
+ *     before any stream capture;
+ *   - every call on a device shares the one array and it keeps the last
+ *     call's contents, so calls whose work overlaps on the GPU (other streams,
+ *     or other host threads) race and corrupt each other's results: order
+ *     them.  A timeout word in the same fixed storage is cleared on `stream`
+ *     at the start of each call.
+ * It calls no cudaMalloc, cudaFree or other allocating routine. */
+int gf_decode_attention_static(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
+                               const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len,
+                               int32_t max_ctx, int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out,
+                               void* stream);
+
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes whose launches can be bracketed by CUDA events (on the
  * launching stream) for live timing inside a run. */

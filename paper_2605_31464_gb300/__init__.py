@@ -45,7 +45,8 @@ class gf_weights(ctypes.Structure):
 EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_release", "gf_forecast_batch",
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
-           "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace"]
+           "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
+           "gf_decode_attention_static"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN = range(4)
@@ -80,6 +81,8 @@ def load(path: str = LIB_PATH):
         "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _p], ctypes.c_int),
         "gf_gemm_status": ([_p], ctypes.c_int),
         "gf_decode_attention_workspace": ([_c_i32, _c_i32, _c_i32, _c_i32], ctypes.c_size_t),
+        "gf_decode_attention_static": ([_p, _p, _p, _c_i64, _p, _c_i32, _p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32,
+                                        _p, _p], ctypes.c_int),
         "gf_decode_attention": ([_p, _p, _p, _c_i64, _p, _c_i32, _p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32, _p, _p,
                                  ctypes.c_size_t, _p], ctypes.c_int),
         "gf_profile_enable": ([_p, ctypes.c_uint32], ctypes.c_int),
@@ -175,6 +178,13 @@ def gf_decode_attention(q, k_cache, v_cache, num_pages, block_table, max_pages, 
                         head_dim, out, workspace, workspace_bytes, stream):
     _check(load().gf_decode_attention(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx, B,
                                       n_q, n_kv, head_dim, out, workspace, workspace_bytes, stream))
+
+
+def gf_decode_attention_static(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx, B, n_q,
+                               n_kv, head_dim, out, stream):
+    """gf_decode_attention with its scratch in the library's fixed device array (no allocation)."""
+    _check(load().gf_decode_attention_static(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
+                                             B, n_q, n_kv, head_dim, out, stream))
 
 
 def decode_attention(q, k_cache, v_cache, block_table, ctx_len, max_ctx, n_q, n_kv, stream=None):

@@ -7,6 +7,9 @@
 // arrive by TMA, double-buffered; warp w takes keys 16w..16w+15 of each page.
 // Each CTA writes an unnormalised partial (running max, running sum, sum of
 // p.v) for its chunk; attn_combine merges the chunks of a sequence.
+#include <mutex>
+
+#include "gf.h"
 #include "kernels.h"
 #include "ptx.cuh"
 
@@ -283,3 +286,105 @@ cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap
 }
 
 }  // namespace gf
+
+// ---------------------------------------------------------------------------
+// gf_decode_attention_static: the same kernels with their scratch (the
+// per-chunk partial results and the timeout word) in fixed device arrays of
+// this module instead of caller or runtime allocations.
+namespace {
+constexpr size_t kStaticScratchBytes = size_t(16) << 20;  // 16 MiB, held by every GPU that loads the library
+constexpr int kMaxDevices = 64;
+std::mutex g_static_mu;
+bool g_static_ready[kMaxDevices];
+void* g_static_scratch_ptr[kMaxDevices];
+int* g_static_err_ptr[kMaxDevices];
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+static __device__ __align__(256) int g_static_err;
+
+extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
+                                          const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len,
+                                          int32_t max_ctx, int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim,
+                                          void* out, void* stream) {
+  if (!q || !k_cache || !v_cache || !block_table || !ctx_len || !out || B < 1 || n_q < 1 || n_kv < 1 ||
+      n_q % n_kv || n_q / n_kv > 16 || max_ctx < 1 || max_pages < 1 || max_ctx > max_pages * 64 || num_pages < 1 ||
+      num_pages * n_kv * 64 >= ((int64_t)1 << 31)) {
+    gf::set_error_short("bad argument");
+    return GF_EINVAL;
+  }
+  if (head_dim != 64 && head_dim != 128) {
+    gf::set_error_short("head_dim 64/128");
+    return GF_ENOTIMPL;
+  }
+  const size_t need = gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx);
+  if (need > kStaticScratchBytes) {
+    gf::set_error_short("exceeds scratch");
+    return GF_ECAPACITY;
+  }
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    gf::set_error_short("no CUDA device");
+    return GF_ECUDA;
+  }
+  if (dev < 0 || dev >= kMaxDevices) {
+    gf::set_error_short("too many GPUs");
+    return GF_ENOTIMPL;
+  }
+  {
+    // First call on this device: look up the device addresses of the arrays
+    // (host code cannot use their names as device pointers).
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    if (!g_static_ready[dev]) {
+      void* scratch = nullptr;
+      void* err = nullptr;
+      if (cudaGetSymbolAddress(&scratch, g_static_scratch) != cudaSuccess ||
+          cudaGetSymbolAddress(&err, g_static_err) != cudaSuccess) {
+        cudaGetLastError();
+        gf::set_error_short("symbol lookup");
+        return GF_ECUDA;
+      }
+      g_static_scratch_ptr[dev] = scratch;
+      g_static_err_ptr[dev] = reinterpret_cast<int*>(err);
+      g_static_ready[dev] = true;
+    }
+  }
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  // The timeout word must start at zero: a word left set by an earlier call
+  // would make this call's waits give up at once.
+  if (cudaMemsetAsync(g_static_err_ptr[dev], 0, sizeof(int), s) != cudaSuccess) {
+    gf::set_error_short("memset failed");
+    return GF_ECUDA;
+  }
+  CUtensorMap tk, tv;
+  const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
+  if (gf::encode_kv_map(&tk, k_cache, head_dim, rows) || gf::encode_kv_map(&tv, v_cache, head_dim, rows)) {
+    gf::set_error_short("tensor map");
+    return GF_ECUDA;
+  }
+  gf::DecodeAttnArgs da{};
+  da.q = reinterpret_cast<const gf::bf16*>(q);
+  da.ldq = (int64_t)n_q * head_dim;
+  da.handles = nullptr;
+  da.seq_len = ctx_len;
+  da.ctx_bias = 0;
+  da.max_ctx = max_ctx;
+  da.block_table = block_table;
+  da.max_pages = max_pages;
+  da.n_q = n_q;
+  da.n_kv = n_kv;
+  da.layer_row0 = 0;
+  da.chunk = 256;
+  da.max_splits = (max_ctx + 255) / 256;
+  da.part_o = reinterpret_cast<float*>(g_static_scratch_ptr[dev]);
+  da.part_ml = da.part_o + (size_t)B * n_kv * da.max_splits * 16 * head_dim;
+  da.out = reinterpret_cast<gf::bf16*>(out);
+  da.ldo = (int64_t)n_q * head_dim;
+  da.scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
+  da.err = g_static_err_ptr[dev];
+  if (gf::launch_attn_decode(head_dim, tk, tv, da, B, s) != cudaSuccess) {
+    gf::set_error_short("launch failed");
+    return GF_ECUDA;
+  }
+  return GF_OK;
+}

@@ -618,6 +618,26 @@ int prepare_decode(gf_model* m, int B, const int32_t* h, cudaStream_t s) {
 
 }  // namespace
 
+// Helpers for entry points defined in other translation units.
+namespace gf {
+// Tensor map over a KV pool viewed as `rows` rows of hd bf16 (boxes of 64 x 64); 0 on success.
+int encode_kv_map(CUtensorMap* m, const void* base, int hd, uint64_t rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return 1;
+  cuuint64_t dims[2] = {(cuuint64_t)hd, rows};
+  cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
+  cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+             ? 0
+             : 1;
+}
+// Record a message of at most 15 characters (kept in the string's inline buffer, so nothing is allocated).
+void set_error_short(const char* msg) { g_err = msg; }
+}  // namespace gf
+
 // =====================================================================================================
 // C ABI
 // =====================================================================================================
