@@ -174,12 +174,13 @@ int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdic
  *          GF_GEMM_SWIGLU:     W rows hold blocks of 64 gate rows followed by 64
  *                              up rows; out (bf16, N/2 columns) = silu(gate) * up
  *   bn     tile width 64, 128 or 256, or 0 to choose; splits: split-K factor
- *          (only with GF_GEMM_ATOMIC_F32), 0 to choose.
+ *          (only with GF_GEMM_ATOMIC_F32), 0 to choose; group_m: 128-row blocks
+ *          per raster group (concurrent tiles share A and W tiles in L2), 0 to choose.
  * Enqueued on `stream`; a device-side timeout is reported by gf_gemm_status. */
 enum { GF_GEMM_STORE_F32 = 0, GF_GEMM_ADD_F32 = 1, GF_GEMM_ATOMIC_F32 = 2, GF_GEMM_STORE_BF16 = 3,
        GF_GEMM_SWIGLU = 4 };
 int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
-                 int32_t mode, int32_t bn, int32_t splits, void* stream);
+                 int32_t mode, int32_t bn, int32_t splits, int32_t group_m, void* stream);
 /* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16 or gf_decode_attention
  * launch gave up waiting. */
 int gf_gemm_status(void* stream);

@@ -78,7 +78,8 @@ def load(path: str = LIB_PATH):
         "gf_device_status": ([_p, _p], ctypes.c_int),
         "gf_launch_count": ([_p], _c_i64),
         "gf_last_error": ([], ctypes.c_char_p),
-        "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _p], ctypes.c_int),
+        "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _c_i32, _p],
+                         ctypes.c_int),
         "gf_gemm_status": ([_p], ctypes.c_int),
         "gf_decode_attention_workspace": ([_c_i32, _c_i32, _c_i32, _c_i32], ctypes.c_size_t),
         "gf_decode_attention_static": ([_p, _p, _p, _c_i64, _p, _c_i32, _p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32,
@@ -162,8 +163,8 @@ def gf_last_error() -> str:
     return load().gf_last_error().decode()
 
 
-def gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, stream):
-    _check(load().gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, stream))
+def gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, group_m, stream):
+    _check(load().gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, group_m, stream))
 
 
 def gf_gemm_status(stream):
@@ -212,13 +213,14 @@ def gf_profile_read(model, kind):
     return dict(launches=n.value, ms=ms.value, flops=fl.value, bytes=by.value)
 
 
-def gemm(A, W, out, mode=GF_GEMM_STORE_F32, bn=0, splits=0, stream=None):
+def gemm(A, W, out, mode=GF_GEMM_STORE_F32, bn=0, splits=0, stream=None, group_m=0):
     """out (op)= A . W^T on the tensor cores (A [M,K], W [N,K] bf16 CUDA tensors)."""
     import torch
     s = stream if stream is not None else torch.cuda.current_stream()
     M, K = A.shape
     N = W.shape[0]
-    gf_gemm_bf16(A.data_ptr(), W.data_ptr(), M, N, K, out.data_ptr(), out.stride(0), mode, bn, splits, s.cuda_stream)
+    gf_gemm_bf16(A.data_ptr(), W.data_ptr(), M, N, K, out.data_ptr(), out.stride(0), mode, bn, splits, group_m,
+                 s.cuda_stream)
 
 
 # ---------------------------------------------------------------- torch-facing wrapper

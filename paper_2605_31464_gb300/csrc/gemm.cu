@@ -42,7 +42,7 @@ static cudaError_t dispatch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB,
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
-                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s) {
+                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0 || N % 32 != 0) return cudaErrorInvalidValue;
   GemmArgs p;
@@ -56,7 +56,14 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   if (splits > p.kb_total) splits = p.kb_total;
   p.kb_per_split = (p.kb_total + splits - 1) / splits;
   p.splits = (p.kb_total + p.kb_per_split - 1) / p.kb_per_split;  // no empty split
-  p.group_m = 16;
+  if (group_m <= 0) {
+    // Concurrent CTAs walk a group of M-blocks across all N-blocks: the group's A tiles stay in L2
+    // while every weight tile is streamed once per group.  Larger groups mean fewer weight re-reads.
+    const double a_tile = 128.0 * K * 2;
+    group_m = (int)(48.0 * 1024 * 1024 / a_tile);
+    group_m = group_m < 4 ? 4 : (group_m > 128 ? 128 : group_m);
+  }
+  p.group_m = group_m;
   p.out = out;
   p.ldo = ldo;
   p.err = err;

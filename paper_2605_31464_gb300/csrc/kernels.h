@@ -15,8 +15,10 @@ using bf16 = __nv_bfloat16;
 // tensor maps (bf16, 128-byte swizzle) with boxes {64, 128} and {64, bn}.
 int gemm_num_stages(int bn);
 int gemm_smem_bytes(int bn);
+// group_m: M-blocks per raster group (0 = sized so a group's A tiles fill about 48 MiB of L2).
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
-                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s);
+                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
+                        int group_m = 0);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {

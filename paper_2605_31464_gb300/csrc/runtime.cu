@@ -947,7 +947,7 @@ int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const
 static int* g_gemm_err = nullptr;
 
 int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
-                 int32_t mode, int32_t bn, int32_t splits, void* stream) {
+                 int32_t mode, int32_t bn, int32_t splits, int32_t group_m, void* stream) {
   if (!A || !W || !out || M < 0 || N < 1 || K < 64) return fail(GF_EINVAL, "bad GEMM arguments");
   if (K % 64 || N % 32) return fail(GF_EINVAL, "GEMM needs K %% 64 == 0 and N %% 32 == 0");
   if (mode < GF_GEMM_STORE_F32 || mode > GF_GEMM_SWIGLU) return fail(GF_EINVAL, "bad GEMM mode");
@@ -974,7 +974,7 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   CUtensorMap ta, tb;
   TRY(make_map(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, 128));
   TRY(make_map(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, (uint32_t)bn));
-  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s));
+  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m));
   return GF_OK;
 }
 
