@@ -162,16 +162,25 @@ def swiglu_ffn(h: np.ndarray, w_gate: np.ndarray, w_up: np.ndarray, w_down: np.n
     return (silu(h @ w_gate.T) * (h @ w_up.T)) @ w_down.T
 
 
+def q_proj(x: np.ndarray, lw: dict, shape: synth.ModelShape, positions: np.ndarray) -> np.ndarray:
+    """Queries of the tokens x at `positions`: RMSNorm, W_q, RoPE.  [T, n_q, hd]"""
+    h = rms_norm(x, lw["attn_norm"], shape.rms_eps)
+    q = (h @ lw["wq"].T).reshape(x.shape[0], shape.n_q, shape.head_dim)
+    return rope(q, positions, shape.rope_theta)
+
+
+def kv_proj(x: np.ndarray, lw: dict, shape: synth.ModelShape, positions: np.ndarray):
+    """Keys (rotated) and values of the tokens x at `positions`.  [T, n_kv, hd] each."""
+    h = rms_norm(x, lw["attn_norm"], shape.rms_eps)
+    k = (h @ lw["wk"].T).reshape(x.shape[0], shape.n_kv, shape.head_dim)
+    v = (h @ lw["wv"].T).reshape(x.shape[0], shape.n_kv, shape.head_dim)
+    return rope(k, positions, shape.rope_theta), v
+
+
 def qkv(x: np.ndarray, lw: dict, shape: synth.ModelShape, positions: np.ndarray):
     """Pre-attention half of a layer for the tokens x: norm, projections, RoPE."""
-    t = x.shape[0]
-    h = rms_norm(x, lw["attn_norm"], shape.rms_eps)
-    q = (h @ lw["wq"].T).reshape(t, shape.n_q, shape.head_dim)
-    k = (h @ lw["wk"].T).reshape(t, shape.n_kv, shape.head_dim)
-    v = (h @ lw["wv"].T).reshape(t, shape.n_kv, shape.head_dim)
-    q = rope(q, positions, shape.rope_theta)
-    k = rope(k, positions, shape.rope_theta)
-    return q, k, v
+    k, v = kv_proj(x, lw, shape, positions)
+    return q_proj(x, lw, shape, positions), k, v
 
 
 def attn_out_and_ffn(x: np.ndarray, a: np.ndarray, lw: dict, shape: synth.ModelShape) -> np.ndarray:
@@ -204,15 +213,15 @@ def layer_forward(x: np.ndarray, lw: dict, shape: synth.ModelShape, positions: n
 def layer_rows(x_all: np.ndarray, lw: dict, shape: synth.ModelShape, rows) -> np.ndarray:
     """One layer's output at selected positions of a single sequence.
 
-    x_all: the layer's input for positions 0..T-1 ([T, d]).  Only the keys
-    and values of positions <= max(rows) are formed; queries and the
-    feed-forward block are evaluated at ``rows`` alone.  Equal, row for row,
-    to layer_forward(x_all, ...)[0][rows].
+    x_all: the layer's input for positions 0..T-1 ([T, d]).  Keys and values
+    are formed for positions <= max(rows); queries and the feed-forward block
+    are evaluated at ``rows`` alone.  Equal, row for row, to
+    layer_forward(x_all, ...)[0][rows].
     """
     rows = np.asarray(rows, dtype=np.int64)
     hi = int(rows.max()) + 1
-    _, k, v = qkv(x_all[:hi], lw, shape, np.arange(hi))
-    q, _, _ = qkv(x_all[rows], lw, shape, rows)
+    k, v = kv_proj(x_all[:hi], lw, shape, np.arange(hi))
+    q = q_proj(x_all[rows], lw, shape, rows)
     a = attention(q, k, v, rows, np.arange(hi))
     return attn_out_and_ffn(x_all[rows], a, lw, shape)
 

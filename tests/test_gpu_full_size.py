@@ -1,0 +1,137 @@
+"""Parity at the full workload sizes, in the launch configuration bench.py uses.
+
+The oracle cannot run a whole 7B/14B forward pass in seconds, so these tests
+compare outputs it can compute one by one.  The whole batch is prefilled at
+its full size through gf_prefill and decoded through gf_decode_step (the
+kernels, tile plans and split factors gf_forecast_batch uses); the GPU's
+residual stream is captured entering and leaving sampled layers, and the
+oracle recomputes those layers from the captured input at sampled rows
+(teacher-forced at layer level).  Also checked: the rotated keys and values
+the GPU cached at sampled positions, the final logits of sampled items
+(from the captured final hidden state), the last decode step of the full
+n_decode run (layer outputs from the GPU's own cache), greedy agreement,
+and the verdict/defer step on the whole batch's final logits.
+
+Layer outputs must match within 2 % of the layer's largest update on that
+row (the update o - x is what bf16 rounding inside the layer perturbs);
+keys/values within bf16 rounding; logits and verdict within the standard
+tolerances.
+"""
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from _helpers import check_logits, check_verdict, greedy_agrees, make_model
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+LAYER_TOL = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2605_31464_gb300 import _build
+    _build.build()
+    assert torch.cuda.is_available()
+
+
+def check_layer(got, ref, x_in, what):
+    upd = np.abs(ref - x_in).max(axis=-1, keepdims=True)
+    err = np.abs(np.asarray(got, dtype=np.float64) - ref)
+    ratio = (err / (upd + 1e-30)).max()
+    assert ratio <= LAYER_TOL, f"{what}: max error {err.max():.3g} = {ratio:.3g} of the layer update"
+    return ratio
+
+
+def check_kv(got_bf16, ref, what):
+    g = got_bf16.float().cpu().numpy().astype(np.float64)
+    err = np.abs(g - ref)
+    bound = 1e-2 * np.abs(ref) + 2e-2 * np.abs(ref).max()
+    assert (err <= bound).all(), f"{what}: max error {err.max():.3g} (scale {np.abs(ref).max():.3g})"
+
+
+def sample_rows(n, seed):
+    base = {0, 1, n // 2, n - 2, n - 1}
+    rng = np.random.default_rng(seed)
+    base |= set(rng.integers(0, n, 3).tolist())
+    return sorted(r for r in base if 0 <= r < n)
+
+
+@pytest.mark.parametrize("name", ["1p5b", "7b_prefill", "7b_decode", "14b_long"])
+def test_full_size_workload(name):
+    import paper_2605_31464_gb300 as gf
+    w = synth.workload(name)
+    m = w.model
+    ids, off = synth.packed_prompts(w)
+    lens = np.diff(off)
+    B, L = w.batch, m.layers
+    model = make_model(m, max_batch=B, max_seq=int(lens.max()) + w.n_decode,
+                       max_prefill_tokens=int(off[-1]))
+    Wo = oracle.Weights(m, cache_layers=False)
+    a = int(np.argmax(lens))            # longest prompt
+    b = int(np.argmin(lens)) if w.ragged else B - 1
+    plan = [(a, 0), (a, L - 1), (b, L // 2)]
+    caps = {}
+    for item, l in plan:
+        for ll in (l, l + 1):
+            if (item, ll) not in caps:
+                caps[(item, ll)] = model.capture(ll, item, int(lens[item]))
+    handles, logits, nxt = model.prefill(torch.from_numpy(ids).cuda(), off)
+    torch.cuda.synchronize()
+    model.status()
+
+    # ---- prefill: sampled layers, cached keys/values, final logits
+    for item, l in plan:
+        n = int(lens[item])
+        x_in = caps[(item, l)].cpu().numpy().astype(np.float64)
+        x_out = caps[(item, l + 1)].cpu().numpy()
+        rows = sample_rows(n, seed=l)
+        lw = Wo.layer(l)
+        ref = oracle.layer_rows(x_in, lw, m, rows)
+        check_layer(x_out[rows], ref, x_in[rows], f"{name} prefill layer {l} item {item}")
+        k_ref, v_ref = oracle.kv_proj(x_in[rows], lw, m, np.array(rows))
+        k_gpu, v_gpu = model.read_kv(l, int(handles[item]), 0, n)
+        check_kv(k_gpu[rows], k_ref, f"{name} cached K layer {l}")
+        check_kv(v_gpu[rows], v_ref, f"{name} cached V layer {l}")
+    h_final = caps[(a, L)].cpu().numpy().astype(np.float64)
+    ref_logits = oracle.lm_head(h_final[-1:], Wo)[0]
+    lg0 = logits[a].cpu().numpy()
+    check_logits(lg0, ref_logits, f"{name} prefill logits item {a}")
+    assert greedy_agrees(int(nxt[a]), ref_logits)
+
+    # ---- the full decode run; checks at its last step
+    toks = nxt
+    for _ in range(w.n_decode - 1):
+        _, toks = model.decode_step(handles, toks, want_logits=False)
+    dec_plan = [(a, 0), (a, L - 1)]
+    dcaps = {}
+    for item, l in dec_plan:
+        for ll in (l, l + 1):
+            dcaps[(item, ll)] = model.capture(ll, item, 1)
+    lg, nx = model.decode_step(handles, toks)
+    torch.cuda.synchronize()
+    model.status()
+    pos = int(lens[a]) + w.n_decode - 1
+    for item, l in dec_plan:
+        x_in = dcaps[(item, l)].cpu().numpy().astype(np.float64)
+        k_prev, v_prev = model.read_kv(l, int(handles[item]), 0, pos)
+        kp = k_prev.float().cpu().numpy().astype(np.float64)
+        vp = v_prev.float().cpu().numpy().astype(np.float64)
+        ref, _, _ = oracle.layer_forward(x_in, Wo.layer(l), m, np.array([pos]), kp, vp)
+        check_layer(dcaps[(item, l + 1)].cpu().numpy(), ref, x_in, f"{name} decode layer {l} at position {pos}")
+    ref_logits = oracle.lm_head(dcaps[(a, L)].cpu().numpy().astype(np.float64), Wo)[0]
+    check_logits(lg[a].cpu().numpy(), ref_logits, f"{name} decode logits at position {pos}")
+    assert greedy_agrees(int(nx[a]), ref_logits)
+
+    # ---- verdict and defer on the whole batch's final logits
+    p, conf, arg, defer = gf.verdict(lg, w.verdict_ids, w.tau)
+    rp, rc, ra, rd = oracle.verdict(lg.cpu().numpy().astype(np.float64), w.verdict_ids, w.tau)
+    p, conf, arg, defer = p.cpu().numpy(), conf.cpu().numpy(), arg.cpu().numpy(), defer.cpu().numpy()
+    for i in range(B):
+        check_verdict(p[i], conf[i], arg[i], defer[i], rp[i], rc[i], ra[i], rd[i], w.tau)
+    model.release(handles)
+    model.close()
+    del model
+    torch.cuda.empty_cache()
