@@ -164,9 +164,10 @@ cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cuda
 }
 
 // ------------------------------------------------------------------ greedy arg max
-// out[b] = arg max_v logits[b, v], lowest v on ties; optionally also out2[b*stride].
+// out[b] = arg max_v logits[b, v], lowest v on ties; optionally also
+// out2[b*stride + col] with col = col_base (+ *step when step is given), if col < col_limit.
 __global__ void argmax_kernel(const float* logits, int64_t ld, int V, int32_t* out, int32_t* out2,
-                              int64_t out2_stride) {
+                              int64_t out2_stride, const int32_t* step, int col_base, int col_limit) {
   const int b = blockIdx.x;
   const float* row = logits + (int64_t)b * ld;
   float best = -INFINITY;
@@ -211,14 +212,17 @@ __global__ void argmax_kernel(const float* logits, int64_t ld, int V, int32_t* o
     if (lane == 0) {
       if (best_i == 0x7fffffff) best_i = 0;  // all NaN: fall back to id 0
       out[b] = best_i;
-      if (out2) out2[(int64_t)b * out2_stride] = best_i;
+      if (out2) {
+        const int col = col_base + (step ? *step : 0);
+        if (col < col_limit) out2[(int64_t)b * out2_stride + col] = best_i;
+      }
     }
   }
 }
 cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
-                          int64_t out2_stride, cudaStream_t s) {
+                          int64_t out2_stride, cudaStream_t s, const int32_t* step, int col_base, int col_limit) {
   if (B <= 0) return cudaSuccess;
-  argmax_kernel<<<B, 1024, 0, s>>>(logits, ld, V, out, out2, out2_stride);
+  argmax_kernel<<<B, 1024, 0, s>>>(logits, ld, V, out, out2, out2_stride, step, col_base, col_limit);
   return cudaGetLastError();
 }
 
@@ -278,13 +282,15 @@ cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int
   return cudaGetLastError();
 }
 
-__global__ void advance_kernel(const int32_t* handles, int B, int32_t* seq_len) {
+// seq_len[handles[b]] += 1 for every b; *step += 1 when step is given (decode-step counter).
+__global__ void advance_kernel(const int32_t* handles, int B, int32_t* seq_len, int32_t* step) {
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) seq_len[handles[b]] += 1;
+  if (step && b == 0) *step += 1;
 }
-cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s) {
+cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s, int32_t* step) {
   if (B <= 0) return cudaSuccess;
-  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(handles, B, seq_len);
+  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(handles, B, seq_len, step);
   return cudaGetLastError();
 }
 

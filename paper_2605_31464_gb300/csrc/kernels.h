@@ -89,12 +89,14 @@ cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, 
                            float eps, bf16* y, int64_t ldy, cudaStream_t s);
 cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s);
 cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
-                          int64_t out2_stride, cudaStream_t s);
+                          int64_t out2_stride, cudaStream_t s, const int32_t* step = nullptr, int col_base = 0,
+                          int col_limit = 1 << 30);
 cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t* ids, int K, float tau, float* p,
                            float* conf, int32_t* arg, uint8_t* defer, cudaStream_t s);
 cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
                                cudaStream_t s);
-cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s);
+cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s,
+                           int32_t* step = nullptr);
 cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                  const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
                                  cudaStream_t s);

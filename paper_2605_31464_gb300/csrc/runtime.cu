@@ -201,6 +201,14 @@ struct gf_model {
   std::vector<cudaEvent_t> ev_pool;
   void* host_out = nullptr;
   size_t host_out_cap = 0;
+  // greedy tokens of gf_forecast_batch: [B_max][tok_stride], column = decode step input index
+  int32_t* tok_hist = nullptr;
+  int tok_stride = 0;
+  int32_t* ctl = nullptr;  // [0]: device decode-step counter
+  // one CUDA graph per batch size for the decode step of gf_forecast_batch
+  cudaStream_t cap_stream = nullptr;
+  std::map<int, cudaGraphExec_t> graphs;
+  int64_t graph_launches_per_step = 0;
 };
 
 namespace {
@@ -511,15 +519,19 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
 
 // One decode step for B live sequences whose handles are already on the
 // device in m->handles (host copy in `h`).
+// With `step` (a device counter), the generated token is also written to
+// tokens_col[b * tokens_stride + *step + 1] and the counter advanced, so that
+// the step can be captured once in a CUDA graph and replayed.
 int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float* logits_dst, int32_t* next_dst,
-                int32_t* tokens_col, int64_t tokens_stride, cudaStream_t s) {
+                int32_t* tokens_col, int64_t tokens_stride, cudaStream_t s, int32_t* step = nullptr,
+                bool capturing = false) {
   CU(gf::launch_embed(ids, B, m->embed, m->vocab, m->d, m->dres, m->err, s));
   m->launches++;
   CU(cudaMemsetAsync(m->dqkv, 0, (size_t)B * m->qkv_dim * sizeof(float), s));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)m->hd);
   for (int l = 0; l < m->L; ++l) {
     const gf_model::Layer& W = m->layers[l];
-    TRY(fire_captures(m, l, m->dres, nullptr, B, true, s));
+    if (!capturing) TRY(fire_captures(m, l, m->dres, nullptr, B, true, s));
     CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, W.attn_norm, m->cfg.rms_eps, m->dxn, m->d, s));
     m->launches++;
     TRY(gemm(m, m->dxn, B, m->d, W.qkv, m->qkv_dim, m->dqkv, m->qkv_dim, gf::kAtomicF32, s, true));
@@ -578,18 +590,62 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     TRY(gemm(m, m->dxn, B, m->d, W.gu, 2 * m->ffn_pad, m->dact, m->ffn_pad, gf::kSwiGLU, s, true, 2 * m->ffn));
     TRY(gemm(m, m->dact, B, m->ffn_pad, W.down, m->d, m->dres, m->d, gf::kAtomicF32, s, true, 0, m->ffn));
   }
-  TRY(fire_captures(m, m->L, m->dres, nullptr, B, true, s));
+  if (!capturing) TRY(fire_captures(m, m->L, m->dres, nullptr, B, true, s));
   CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
   m->launches++;
   float* lg = logits_dst ? logits_dst : m->logits;
   TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, true));
   if (next_dst) {
-    CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+    if (step)
+      CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s, step, 1,
+                           (int)tokens_stride));
+    else
+      CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
     m->launches++;
   }
-  CU(gf::launch_advance(m->handles, B, m->seq_len, s));
+  CU(gf::launch_advance(m->handles, B, m->seq_len, s, step));
   m->launches++;
-  for (int b = 0; b < B; ++b) m->h_len[h[b]] += 1;
+  if (!capturing)
+    for (int b = 0; b < B; ++b) m->h_len[h[b]] += 1;
+  return GF_OK;
+}
+
+// The decode step of gf_forecast_batch for a batch of B sequences whose
+// handles are in m->handles, captured once as a CUDA graph: ids and tokens
+// come from m->next, logits go to m->logits, generated tokens to m->tok_hist.
+int decode_graph(gf_model* m, int B, const int32_t* h, cudaGraphExec_t* out) {
+  auto it = m->graphs.find(B);
+  if (it != m->graphs.end()) {
+    *out = it->second;
+    return GF_OK;
+  }
+  if (!m->cap_stream) CU(cudaStreamCreateWithFlags(&m->cap_stream, cudaStreamNonBlocking));
+  const uint32_t mask = m->prof_mask;
+  m->prof_mask = 0;
+  const int64_t launches = m->launches;
+  CU(cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal));
+  int rc = decode_impl(m, B, h, m->next, m->logits, m->next, m->tok_hist, m->tok_stride, m->cap_stream, m->ctl,
+                       true);
+  cudaGraph_t g = nullptr;
+  const cudaError_t e = cudaStreamEndCapture(m->cap_stream, &g);
+  m->prof_mask = mask;
+  m->graph_launches_per_step = m->launches - launches;
+  m->launches = launches;
+  if (rc != GF_OK) {
+    if (g) cudaGraphDestroy(g);
+    return rc;
+  }
+  if (e != cudaSuccess) return fail(GF_ECUDA, "decode-step capture failed: %s", cudaGetErrorString(e));
+  cudaGraphExec_t exec = nullptr;
+  const cudaError_t e2 = cudaGraphInstantiate(&exec, g, 0);
+  cudaGraphDestroy(g);
+  if (e2 != cudaSuccess) return fail(GF_ECUDA, "graph instantiation failed: %s", cudaGetErrorString(e2));
+  if (m->graphs.size() >= 16) {
+    for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+    m->graphs.clear();
+  }
+  m->graphs[B] = exec;
+  *out = exec;
   return GF_OK;
 }
 
@@ -650,6 +706,8 @@ int64_t gf_launch_count(const gf_model* m) { return m ? m->launches : 0; }
 void gf_destroy(gf_model* m) {
   if (!m) return;
   cudaDeviceSynchronize();
+  for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
+  if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
   m->staging.release();
   for (void* p : m->allocs) cudaFree(p);
   if (m->host_out) cudaFreeHost(m->host_out);
@@ -752,6 +810,9 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->fcall, 3 * Bm + 8);
   if (!rc) rc = dalloc(m, &m->out_small, Bm * 12);
   if (!rc) rc = dalloc(m, &m->err, 1);
+  m->tok_stride = c.max_seq;
+  if (!rc) rc = dalloc(m, &m->tok_hist, Bm * m->tok_stride);
+  if (!rc) rc = dalloc(m, &m->ctl, 4);
   if (rc) return bail(rc);
 
   // ---- pack weights
@@ -876,16 +937,35 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
   m->launches++;
   std::vector<int32_t> h(B);
   float* lg = (n_decode == 0 && final_logits) ? final_logits : m->logits;
-  // tokens[b, s] is the input of decode step s: the arg max of the logits before it
-  TRY(prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), lg, m->next, s,
-                   (tokens && n_decode > 0) ? tokens : nullptr, n_decode));
+  // tok_hist[b, s] is the input of decode step s: the arg max of the logits before it
+  TRY(prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), lg, m->next, s, m->tok_hist,
+                   m->tok_stride));
   int rc = upload(m->staging, m->handles, h.data(), (size_t)B * sizeof(int32_t), s);
-  for (int step = 0; step < n_decode && rc == GF_OK; ++step) {
-    float* dst = (step == n_decode - 1 && final_logits) ? final_logits : m->logits;
-    lg = dst;
-    int32_t* col = (tokens && step + 1 < n_decode) ? tokens + step + 1 : nullptr;
-    rc = decode_impl(m, B, h.data(), m->next, dst, m->next, col, n_decode, s);
+  if (rc == GF_OK && n_decode > 0) {
+    lg = m->logits;
+    if (cudaMemsetAsync(m->ctl, 0, sizeof(int32_t), s) != cudaSuccess) rc = fail(GF_ECUDA, "memset failed");
+    // the first step runs eagerly (it also configures the kernels); the rest replay one captured graph
+    if (rc == GF_OK) rc = decode_impl(m, B, h.data(), m->next, m->logits, m->next, m->tok_hist, m->tok_stride, s, m->ctl);
+    if (rc == GF_OK && n_decode > 1) {
+      cudaGraphExec_t exec = nullptr;
+      rc = decode_graph(m, B, h.data(), &exec);
+      for (int step = 1; step < n_decode && rc == GF_OK; ++step) {
+        const cudaError_t e = cudaGraphLaunch(exec, s);
+        if (e != cudaSuccess) rc = fail(GF_ECUDA, "graph launch failed: %s", cudaGetErrorString(e));
+        m->launches += m->graph_launches_per_step;
+      }
+      if (rc == GF_OK)
+        for (int b = 0; b < B; ++b) m->h_len[h[b]] += n_decode - 1;
+    }
+    if (rc == GF_OK && final_logits &&
+        cudaMemcpyAsync(final_logits, m->logits, (size_t)B * m->vocab * sizeof(float), cudaMemcpyDeviceToDevice,
+                        s) != cudaSuccess)
+      rc = fail(GF_ECUDA, "logits copy failed");
   }
+  if (rc == GF_OK && tokens && n_decode > 0 &&
+      cudaMemcpy2DAsync(tokens, (size_t)n_decode * sizeof(int32_t), m->tok_hist, (size_t)m->tok_stride * sizeof(int32_t),
+                        (size_t)n_decode * sizeof(int32_t), B, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    rc = fail(GF_ECUDA, "tokens copy failed");
   if (rc == GF_OK) {
     const cudaError_t e = gf::launch_verdict(lg, m->vocab, B, verdict_ids, K, tau, p, conf, verdict_arg, defer, s);
     if (e != cudaSuccess) rc = fail(GF_ECUDA, "verdict launch: %s", cudaGetErrorString(e));
