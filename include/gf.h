@@ -190,7 +190,9 @@ int gf_gemm_status(void* stream);
  *   out[b, h, :] = sum_j softmax_j(q[b,h,:] . k_j / sqrt(hd)) v_j  over the
  *   ctx_len[b] cached positions j of sequence b, kv head h / (n_q / n_kv).
  *   q            device bf16 [B, n_q*hd], already rotated
- *   k_cache, v_cache device bf16 [num_pages][n_kv][64][hd] (64-token pages)
+ *   k_cache      device bf16 [num_pages][n_kv][64][hd] (64-token pages)
+ *   v_cache      device bf16 [num_pages][n_kv][hd][64]: each page stored
+ *                transposed (head dim major, 64 tokens contiguous)
  *   block_table  device int32 [B][max_pages]: page of block j of sequence b
  *   ctx_len      device int32 [B], 1 <= ctx_len[b] <= max_ctx (a larger
  *                value is clamped to max_ctx; 0 gives a zero output row)

@@ -3,8 +3,9 @@
 // Grid (split, kv_head, sequence).  A CTA takes `chunk` keys of one sequence
 // and one KV head and serves every query head of that group at once (the G
 // heads of a GQA group are the 16 rows of a warp MMA, zero-padded), so each
-// K/V page is read from HBM once per step.  Pages (64 tokens x head_dim)
-// arrive by TMA, double-buffered; warp w takes keys 16w..16w+15 of each page.
+// K/V page is read from HBM once per step.  A K page (64 tokens x head_dim)
+// and a V page (stored transposed, head_dim x 64 tokens) arrive by TMA,
+// double-buffered; warp w takes keys 16w..16w+15 of each page.
 // Each CTA writes an unnormalised partial (running max, running sum, sum of
 // p.v) for its chunk; attn_combine merges the chunks of a sequence.
 #include <mutex>
@@ -18,8 +19,8 @@ namespace gf {
 template <int HD>
 struct DecodeCfg {
   static constexpr int HALVES = HD / 64;
-  static constexpr int PAGE_HALF = 64 * 128;        // one 64-column half of a page
-  static constexpr int PAGE_BYTES = 64 * HD * 2;    // one page of K (or V) for one head
+  static constexpr int PAGE_HALF = 64 * 128;        // one 64-column half of a K page
+  static constexpr int PAGE_BYTES = 64 * HD * 2;    // one page of K (or V^T) for one head
   static constexpr int Q_BYTES = 16 * HD * 2;
   // smem: Q [HALVES][16][128 B] | K[2] | V[2] | barriers ; the K/V area is reused to combine warps
   static constexpr int SMEM = 1024 + Q_BYTES + 4 * PAGE_BYTES + 64;
@@ -54,13 +55,12 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
 
   auto issue = [&](int i) {
     const int buf = i & 1;
-    const int64_t row = a.layer_row0 + ((int64_t)pages[p0 + i] * a.n_kv + kvh) * 64;
+    const int64_t pg = (int64_t)pages[p0 + i] * a.n_kv + kvh;
     mbar_arrive_expect_tx(&bar[buf], 2 * C::PAGE_BYTES);
 #pragma unroll
-    for (int h = 0; h < C::HALVES; ++h) {
-      tma_load_2d(sK + buf * C::PAGE_BYTES + h * C::PAGE_HALF, &tmK, &bar[buf], h * 64, (int)row);
-      tma_load_2d(sV + buf * C::PAGE_BYTES + h * C::PAGE_HALF, &tmV, &bar[buf], h * 64, (int)row);
-    }
+    for (int h = 0; h < C::HALVES; ++h)
+      tma_load_2d(sK + buf * C::PAGE_BYTES + h * C::PAGE_HALF, &tmK, &bar[buf], h * 64, (int)(a.layer_row0 + pg * 64));
+    tma_load_2d(sV + buf * C::PAGE_BYTES, &tmV, &bar[buf], 0, (int)(a.layer_vrow0 + pg * HD));
   };
 
   if (threadIdx.x == 0) {
@@ -169,12 +169,13 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
     pa[1] = pack_bf16(s[0][2], s[0][3]);
     pa[2] = pack_bf16(s[1][0], s[1][1]);
     pa[3] = pack_bf16(s[1][2], s[1][3]);
+    // V^T page: row = head dim, 64 keys per 128-byte row; this warp's keys are chunks 2w, 2w+1
 #pragma unroll
     for (int dp = 0; dp < HD / 16; ++dp) {
-      const int key = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-      const int chunk = dp * 2 + (lane >> 4);
+      const int dim = dp * 16 + (lane & 7) + (lane >> 4) * 8;
+      const int chunk = warp * 2 + ((lane >> 3) & 1);
       uint32_t b0, b1, b2, b3;
-      ldsm_x4_t(smem_u32(v_t + (chunk >> 3) * C::PAGE_HALF) + sw128(key, chunk & 7), b0, b1, b2, b3);
+      ldsm_x4(smem_u32(v_t) + sw128(dim, chunk), b0, b1, b2, b3);
       mma_bf16_16816(o[2 * dp], pa, b0, b1);
       mma_bf16_16816(o[2 * dp + 1], pa, b2, b3);
     }
@@ -358,7 +359,8 @@ extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, co
   }
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
-  if (gf::encode_kv_map(&tk, k_cache, head_dim, rows) || gf::encode_kv_map(&tv, v_cache, head_dim, rows)) {
+  if (gf::encode_kv_map(&tk, k_cache, head_dim, rows) ||
+      gf::encode_vt_map(&tv, v_cache, head_dim, (uint64_t)num_pages * n_kv * head_dim)) {
     gf::set_error_short("tensor map");
     return GF_ECUDA;
   }
@@ -374,6 +376,7 @@ extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, co
   da.n_q = n_q;
   da.n_kv = n_kv;
   da.layer_row0 = 0;
+  da.layer_vrow0 = 0;
   da.chunk = 256;
   da.max_splits = (max_ctx + 255) / 256;
   da.part_o = reinterpret_cast<float*>(g_static_scratch_ptr[dev]);

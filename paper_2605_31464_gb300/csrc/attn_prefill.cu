@@ -1,41 +1,70 @@
-// Causal grouped-query attention over the prompt (prefill).
+// Causal grouped-query attention over the prompt (prefill) on the tcgen05
+// tensor cores.
 //
-// One CTA = 128 query rows of one head of one prompt; 8 warps own 16 rows
-// each.  Q (two 64-column halves) and every 64-key K/V tile arrive by TMA
-// with 128-byte swizzling; K/V tiles are read straight from the paged KV
-// cache (a tile is one 64-token page).  Scores and P.V use bf16 warp MMAs with
-// fp32 accumulation and an online (running max / running sum) softmax in the
-// log2 domain; the output is normalised once at the end.
+// One CTA = 128 query rows of one head of one prompt, walking 128-key tiles
+// (two 64-token pages of the paged KV cache) up to the diagonal:
+//   warp 0      TMA producer: Q once; K and V^T tiles into two-deep rings
+//   warp 1      one thread issues S = Q K^T (M 128 x N 128 x K hd) into a
+//               double-buffered TMEM score buffer, and O += P_j V_j (M 128 x
+//               N hd x K 128) into one TMEM accumulator
+//   warps 2..5  softmax: thread r owns query row r (TMEM lane r): loads its
+//               whole score row, writes P_j = exp2(s - m) as bf16 into shared
+//               memory for the P V product and keeps the row sum l.  The
+//               reference max m is raised (and O, l rescaled in place) only
+//               when a tile's max exceeds it by more than 2^8, so O and l
+//               always share the same reference and o = O / l is exact.
+// The V cache is stored transposed per page ([page][kv head][hd][64 keys]) so
+// that both products read K-major operands.  Every wait is bounded.
 #include "kernels.h"
 #include "ptx.cuh"
 
 namespace gf {
 
 template <int HD>
-struct PrefillCfg {
+struct FaCfg {
   static constexpr int BQ = 128;
-  static constexpr int BKV = 64;
-  static constexpr int HALVES = HD / 64;
+  static constexpr int BKV = 128;
+  static constexpr int HALVES = HD / 64;                // 64-column blocks of Q and K
   static constexpr int Q_BYTES = BQ * HD * 2;
-  static constexpr int Q_HALF = BQ * 128;   // bytes of one 64-column half of Q
-  static constexpr int KV_HALF = BKV * 128; // bytes of one 64-column half of a K or V tile
-  static constexpr int KV_BYTES = BKV * HD * 2;
-  static constexpr int SMEM = 1024 + Q_BYTES + 4 * KV_BYTES + 64;
+  static constexpr int K_BYTES = BKV * HD * 2;          // HALVES blocks of [128 keys][64]
+  static constexpr int K_BLOCK = BKV * 128;
+  static constexpr int V_BYTES = HD * BKV * 2;          // 2 page blocks of [HD rows][64 keys]
+  static constexpr int V_BLOCK = HD * 128;
+  static constexpr int P_BYTES = BQ * BKV * 2;          // 2 key blocks of [128 rows][64 keys]
+  static constexpr int P_BLOCK = BQ * 128;
+  static constexpr int SMEM = 1024 + Q_BYTES + 2 * K_BYTES + 2 * V_BYTES + 2 * P_BYTES + 256;
+  // tensor memory: S[2] at columns 0 and 128; the O accumulator at 256
+  static constexpr uint32_t TMEM_COLS = 512;
+  static constexpr uint32_t S_COL = 0;
+  static constexpr uint32_t O_COL = 256;
 };
 
 template <int HD>
-__global__ void __launch_bounds__(256) attn_prefill_kernel(const __grid_constant__ CUtensorMap tmQ,
-                                                           const __grid_constant__ CUtensorMap tmK,
-                                                           const __grid_constant__ CUtensorMap tmV,
-                                                           const PrefillAttnArgs a) {
-  using C = PrefillCfg<HD>;
+__global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_constant__ CUtensorMap tmQ,
+                                                                 const __grid_constant__ CUtensorMap tmK,
+                                                                 const __grid_constant__ CUtensorMap tmV,
+                                                                 const PrefillAttnArgs a) {
+  using C = FaCfg<HD>;
+  constexpr uint32_t IDESC_S = idesc_bf16_f32(128, C::BKV);
+  constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* sQ = smem;                          // [HALVES][128 rows][128 B]
-  uint8_t* sK = sQ + C::Q_BYTES;               // [2 bufs][HALVES][64][128 B]
-  uint8_t* sV = sK + 2 * C::KV_BYTES;
-  uint64_t* bar_q = reinterpret_cast<uint64_t*>(sV + 2 * C::KV_BYTES);
-  uint64_t* bar_kv = bar_q + 1;                // [2]
+  uint8_t* sQ = smem;
+  uint8_t* sK = sQ + C::Q_BYTES;        // [2][K_BYTES]
+  uint8_t* sV = sK + 2 * C::K_BYTES;    // [2][V_BYTES]
+  uint8_t* sP = sV + 2 * C::V_BYTES;    // [2][P_BYTES]
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sP + 2 * C::P_BYTES);
+  uint64_t* q_full = bar;
+  uint64_t* k_full = bar + 1;    // [2]
+  uint64_t* k_empty = bar + 3;   // [2]
+  uint64_t* v_full = bar + 5;    // [2]
+  uint64_t* v_empty = bar + 7;   // [2]
+  uint64_t* s_full = bar + 9;    // [2]
+  uint64_t* s_free = bar + 11;   // [2]
+  uint64_t* p_full = bar + 13;   // [2]
+  uint64_t* o_done = bar + 15;   // [2]: P V of tile j completes phase j/2 of o_done[j % 2]
+  uint64_t* mma_done = bar + 19;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 20);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -46,179 +75,244 @@ __global__ void __launch_bounds__(256) attn_prefill_kernel(const __grid_constant
   const int seq_start = a.offsets[b];
   const int len = a.offsets[b + 1] - seq_start;
   const int kvh = head / (a.n_q / a.n_kv);
-  const int slot = a.slots[b];
-  const int32_t* pages = a.block_table + (int64_t)slot * a.max_pages;
+  const int32_t* pages = a.block_table + (int64_t)a.slots[b] * a.max_pages;
+  const int n_pages = (len + 63) >> 6;
   const int n_tiles = (min(q0 + C::BQ, len) + C::BKV - 1) / C::BKV;
 
-  auto issue_kv = [&](int j) {
-    const int buf = j & 1;
-    const int64_t row = a.layer_row0 + ((int64_t)pages[j] * a.n_kv + kvh) * 64;
-    mbar_arrive_expect_tx(&bar_kv[buf], 2 * C::KV_BYTES);
-#pragma unroll
-    for (int h = 0; h < C::HALVES; ++h) {
-      tma_load_2d(sK + buf * C::KV_BYTES + h * C::KV_HALF, &tmK, &bar_kv[buf], h * 64, (int)row);
-      tma_load_2d(sV + buf * C::KV_BYTES + h * C::KV_HALF, &tmV, &bar_kv[buf], h * 64, (int)row);
-    }
-  };
-
   if (threadIdx.x == 0) {
-    mbar_init(bar_q, 1);
-    mbar_init(&bar_kv[0], 1);
-    mbar_init(&bar_kv[1], 1);
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&k_full[i], 1);
+      mbar_init(&k_empty[i], 1);
+      mbar_init(&v_full[i], 1);
+      mbar_init(&v_empty[i], 1);
+      mbar_init(&s_full[i], 1);
+      mbar_init(&s_free[i], 128);
+      mbar_init(&p_full[i], 128);
+      mbar_init(&o_done[i], 1);
+    }
+    mbar_init(mma_done, 1);
     fence_mbar_init();
     fence_async_smem();
-    mbar_arrive_expect_tx(bar_q, C::Q_BYTES);
-#pragma unroll
-    for (int h = 0; h < C::HALVES; ++h)
-      tma_load_2d(sQ + h * C::Q_HALF, &tmQ, bar_q, head * HD + h * 64, seq_start + q0);
-    issue_kv(0);
-    if (n_tiles > 1) issue_kv(1);
+    prefetch_tmap(&tmQ);
+    prefetch_tmap(&tmK);
+    prefetch_tmap(&tmV);
   }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, C::TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
 
-  bool ok = mbar_wait(bar_q, 0, a.err);
-
-  // Q fragments: rows 16*warp .. +15, all HD columns.
-  uint32_t qa[HD / 16][4];
-  {
-    const int r = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+  if (warp == 0) {
+    // -------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      mbar_arrive_expect_tx(q_full, C::Q_BYTES);
 #pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-      const int chunk = kk * 2 + (lane >> 4);
-      const uint32_t addr = smem_u32(sQ + (chunk >> 3) * C::Q_HALF) + sw128(r, chunk & 7);
-      ldsm_x4(addr, qa[kk][0], qa[kk][1], qa[kk][2], qa[kk][3]);
-    }
-  }
-
-  float o[HD / 8][4];
+      for (int h = 0; h < C::HALVES; ++h)
+        tma_load_2d(sQ + h * C::Q_BYTES / C::HALVES, &tmQ, q_full, head * HD + h * 64, seq_start + q0);
+      int k_issued = 0, v_issued = 0;
+      bool ok = true;
+      for (int j = 0; j < n_tiles && ok; ++j) {
+        const int st = j & 1;
+        const uint32_t ph = ((j >> 1) & 1) ^ 1u;
+        // pages of this 128-key tile; a missing second page re-reads the first (its keys are masked)
+        const int pg0 = pages[2 * j];
+        const int pg1 = (2 * j + 1 < n_pages) ? pages[2 * j + 1] : pg0;
+        if (!mbar_wait(&k_empty[st], ph, a.err)) { ok = false; break; }
+        mbar_arrive_expect_tx(&k_full[st], C::K_BYTES);
 #pragma unroll
-  for (int i = 0; i < HD / 8; ++i) o[i][0] = o[i][1] = o[i][2] = o[i][3] = 0.f;
-  float m_run[2] = {-INFINITY, -INFINITY};
-  float l_run[2] = {0.f, 0.f};
-  const int g = lane >> 2, t4 = lane & 3;
-  const int qpos0 = q0 + warp * 16 + g;  // position of fragment row g; row g+8 is qpos0 + 8
-
-  int j_fail = 0;
-  for (int j = 0; j < n_tiles && ok; ++j) {
-    const int buf = j & 1;
-    if (!mbar_wait(&bar_kv[buf], (j >> 1) & 1, a.err)) {
-      ok = false;
-      j_fail = j;
-      break;
-    }
-    const uint8_t* k_t = sK + buf * C::KV_BYTES;
-    const uint8_t* v_t = sV + buf * C::KV_BYTES;
-    // ---- S = Q K^T (16 x 64 per warp)
-    float s[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i][0] = s[i][1] = s[i][2] = s[i][3] = 0.f;
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-#pragma unroll
-      for (int np = 0; np < 4; ++np) {
-        const int key = np * 16 + (lane & 7) + (lane >> 4) * 8;
-        const int chunk = kk * 2 + ((lane >> 3) & 1);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4(smem_u32(k_t + (chunk >> 3) * C::KV_HALF) + sw128(key, chunk & 7), b0, b1, b2, b3);
-        mma_bf16_16816(s[2 * np], qa[kk], b0, b1);
-        mma_bf16_16816(s[2 * np + 1], qa[kk], b2, b3);
-      }
-    }
-    // ---- mask, online softmax
-    const int key0 = j * C::BKV;
-    const bool need_mask = (key0 + C::BKV - 1 > q0 + warp * 16) || (key0 + C::BKV > len);
-    float mx[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-    for (int n = 0; n < 8; ++n) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        float v = s[n][e] * a.scale_log2;
-        if (need_mask) {
-          const int key = key0 + n * 8 + 2 * t4 + (e & 1);
-          const int qp = qpos0 + (e >> 1) * 8;
-          if (key > qp || key >= len) v = -INFINITY;
+        for (int h = 0; h < C::HALVES; ++h) {
+          uint8_t* dst = sK + st * C::K_BYTES + h * C::K_BLOCK;
+          tma_load_2d(dst, &tmK, &k_full[st], h * 64, (int)(a.layer_row0 + ((int64_t)pg0 * a.n_kv + kvh) * 64));
+          tma_load_2d(dst + 64 * 128, &tmK, &k_full[st], h * 64,
+                      (int)(a.layer_row0 + ((int64_t)pg1 * a.n_kv + kvh) * 64));
         }
-        s[n][e] = v;
-        mx[e >> 1] = fmaxf(mx[e >> 1], v);
+        ++k_issued;
+        if (!mbar_wait(&v_empty[st], ph, a.err)) { ok = false; break; }
+        mbar_arrive_expect_tx(&v_full[st], C::V_BYTES);
+        uint8_t* dv = sV + st * C::V_BYTES;
+        tma_load_2d(dv, &tmV, &v_full[st], 0, (int)(a.layer_vrow0 + ((int64_t)pg0 * a.n_kv + kvh) * HD));
+        tma_load_2d(dv + C::V_BLOCK, &tmV, &v_full[st], 0, (int)(a.layer_vrow0 + ((int64_t)pg1 * a.n_kv + kvh) * HD));
+        ++v_issued;
+      }
+      // copies still in flight must land before the CTA exits
+      mbar_wait_drain(q_full, 0);
+      for (int j = max(0, k_issued - 2); j < k_issued; ++j) mbar_wait_drain(&k_full[j & 1], (j >> 1) & 1);
+      for (int j = max(0, v_issued - 2); j < v_issued; ++j) mbar_wait_drain(&v_full[j & 1], (j >> 1) & 1);
+    }
+  } else if (warp == 1) {
+    // -------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      bool ok = mbar_wait(q_full, 0, a.err);
+      bool any = false;
+      auto issue_s = [&](int j) -> bool {
+        const int st = j & 1;
+        if (!mbar_wait(&k_full[st], (j >> 1) & 1, a.err)) return false;
+        if (!mbar_wait(&s_free[st], ((j >> 1) & 1) ^ 1u, a.err)) return false;
+        tc_fence_after();
+        const uint32_t d = tmem + C::S_COL + st * 128;
+        const uint32_t q_base = smem_u32(sQ), k_base = smem_u32(sK + st * C::K_BYTES);
+#pragma unroll
+        for (int ks = 0; ks < HD / 16; ++ks) {
+          const uint32_t off = (ks & 3) * 32;
+          umma_bf16(d, sdesc_k_sw128(q_base + (ks >> 2) * (C::Q_BYTES / C::HALVES) + off),
+                    sdesc_k_sw128(k_base + (ks >> 2) * C::K_BLOCK + off), IDESC_S, ks > 0 ? 1u : 0u);
+        }
+        umma_commit(&s_full[st]);
+        umma_commit(&k_empty[st]);
+        any = true;
+        return true;
+      };
+      auto issue_o = [&](int j) -> bool {
+        const int st = j & 1;
+        if (!mbar_wait(&v_full[st], (j >> 1) & 1, a.err)) return false;
+        if (!mbar_wait(&p_full[st], (j >> 1) & 1, a.err)) return false;
+        tc_fence_after();
+        const uint32_t d = tmem + C::O_COL;
+        const uint32_t p_base = smem_u32(sP + st * C::P_BYTES), v_base = smem_u32(sV + st * C::V_BYTES);
+#pragma unroll
+        for (int ks = 0; ks < C::BKV / 16; ++ks) {
+          const uint32_t off = (ks & 3) * 32;
+          umma_bf16(d, sdesc_k_sw128(p_base + (ks >> 2) * C::P_BLOCK + off),
+                    sdesc_k_sw128(v_base + (ks >> 2) * C::V_BLOCK + off), IDESC_O, (j > 0 || ks > 0) ? 1u : 0u);
+        }
+        umma_commit(&o_done[st]);
+        umma_commit(&v_empty[st]);
+        return true;
+      };
+      if (ok) ok = issue_s(0);
+      for (int j = 0; j < n_tiles && ok; ++j) {
+        if (j + 1 < n_tiles) ok = issue_s(j + 1);
+        if (ok) ok = issue_o(j);
+      }
+      if (any) {
+        umma_commit(mma_done);
+        mbar_wait_drain(mma_done, 0);
       }
     }
-    float corr[2];
+  } else {
+    // -------------------------------------------------------------- softmax warps 2..5
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // query row within the tile = TMEM lane
+    const int qpos = q0 + r;
+    const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
+    const uint32_t o_addr = tmem + lane_off + C::O_COL;
+    float m_ref = -INFINITY, l_run = 0.f;
+    bool ok = true;
+    // wait until P V of tile t has completed (warp-uniform)
+    auto wait_o = [&](int t) -> bool {
+      return __all_sync(0xffffffffu, mbar_wait(&o_done[t & 1], (t >> 1) & 1, a.err));
+    };
+    for (int j = 0; j < n_tiles && ok; ++j) {
+      const int st = j & 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(&s_full[st], (j >> 1) & 1, a.err))) { ok = false; break; }
+      tc_fence_after();
+      uint32_t v[C::BKV];
+      const uint32_t s_addr = tmem + lane_off + C::S_COL + st * 128;
 #pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 1));
-      mx[r] = fmaxf(mx[r], __shfl_xor_sync(0xffffffffu, mx[r], 2));
-      const float m_new = fmaxf(m_run[r], mx[r]);
-      const float m_use = (m_new == -INFINITY) ? 0.f : m_new;
-      corr[r] = exp2f(m_run[r] - m_use);
-      m_run[r] = m_new;
-      mx[r] = m_use;
+      for (int c = 0; c < C::BKV / 32; ++c) tmem_ld32(s_addr + c * 32, *reinterpret_cast<uint32_t(*)[32]>(&v[c * 32]));
+      tmem_ld_wait();
+      tc_fence_before();
+      mbar_arrive(&s_free[st]);
+      const int key0 = j * C::BKV;
+      // causal / length mask only on the diagonal and last tiles (warp-uniform branch)
+      if ((key0 + C::BKV - 1 > q0) || (key0 + C::BKV > len)) {
+        const int lim = min(qpos + 1, len) - key0;  // keys [0, lim) of this tile are visible
+#pragma unroll
+        for (int i = 0; i < C::BKV; ++i)
+          if (i >= lim) v[i] = __float_as_uint(-INFINITY);
+      }
+      // row max by a tree of independent partial maxima
+      float pm[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) pm[k] = __uint_as_float(v[k]);
+#pragma unroll
+      for (int i = 8; i < C::BKV; ++i) pm[i & 7] = fmaxf(pm[i & 7], __uint_as_float(v[i]));
+      const float mx = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7]))) * a.scale_log2;
+      // raise the reference max (rescaling O and l) only when this tile exceeds it by more than 2^8
+      const bool raise = mx > m_ref + 8.f;
+      if (__any_sync(0xffffffffu, raise)) {
+        const float m_new = raise ? mx : m_ref;
+        const float f = (m_ref == -INFINITY) ? 0.f : exp2f(m_ref - m_new);
+        if (j > 0) {
+          if (!wait_o(j - 1)) { ok = false; break; }
+          tc_fence_after();
+#pragma unroll 1
+          for (int c = 0; c < HD / 32; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(o_addr + c * 32, ov);
+            tmem_ld_wait();
+#pragma unroll
+            for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * f);
+            tmem_st32(o_addr + c * 32, ov);
+          }
+          tmem_st_wait();
+        }
+        l_run *= f;
+        m_ref = m_new;
+      }
+      // the P buffer of this tile was last read by P V of tile j - 2
+      if (j >= 2 && !wait_o(j - 2)) { ok = false; break; }
+      const float neg_m = (m_ref == -INFINITY) ? 0.f : -m_ref;
+      float ps[8];
+#pragma unroll
+      for (int k = 0; k < 8; ++k) ps[k] = 0.f;
+      uint8_t* pbuf = sP + st * C::P_BYTES;
+#pragma unroll
+      for (int c = 0; c < C::BKV / 32; ++c) {
+        uint32_t pk[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+          const float p0 = ex2_approx(fmaf(__uint_as_float(v[c * 32 + i]), a.scale_log2, neg_m));
+          const float p1 = ex2_approx(fmaf(__uint_as_float(v[c * 32 + i + 1]), a.scale_log2, neg_m));
+          ps[(i >> 1) & 7] += p0 + p1;
+          pk[i >> 1] = pack_bf16(p0, p1);
+        }
+        // keys c*32 .. c*32+31 sit in key block c/2, 16-byte chunks (c%2)*4 .. +3 of row r
+        uint8_t* blk = pbuf + (c >> 1) * C::P_BLOCK;
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+          *reinterpret_cast<uint4*>(blk + sw128(r, (c & 1) * 4 + q)) =
+              make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+      }
+      const float rs = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
+      l_run += rs;
+      fence_async_smem();  // P (generic-proxy writes) visible to the tensor core
+      tc_fence_before();
+      mbar_arrive(&p_full[st]);
     }
-    float rs[2] = {0.f, 0.f};
+    if (ok && wait_o(n_tiles - 1)) {
+      tc_fence_after();
+      const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+      uint4* dst = reinterpret_cast<uint4*>(a.out + (int64_t)(seq_start + (qpos < len ? qpos : 0)) * a.ldo + head * HD);
+#pragma unroll 1
+      for (int c = 0; c < HD / 32; ++c) {
+        uint32_t ov[32];
+        tmem_ld32(o_addr + c * 32, ov);
+        tmem_ld_wait();
+        if (qpos < len) {
 #pragma unroll
-    for (int n = 0; n < 8; ++n) {
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const float pv = exp2f(s[n][e] - mx[e >> 1]);
-        s[n][e] = pv;
-        rs[e >> 1] += pv;
+          for (int q = 0; q < 4; ++q)
+            dst[c * 4 + q] = make_uint4(
+                pack_bf16(__uint_as_float(ov[8 * q]) * inv, __uint_as_float(ov[8 * q + 1]) * inv),
+                pack_bf16(__uint_as_float(ov[8 * q + 2]) * inv, __uint_as_float(ov[8 * q + 3]) * inv),
+                pack_bf16(__uint_as_float(ov[8 * q + 4]) * inv, __uint_as_float(ov[8 * q + 5]) * inv),
+                pack_bf16(__uint_as_float(ov[8 * q + 6]) * inv, __uint_as_float(ov[8 * q + 7]) * inv));
+        }
       }
     }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) l_run[r] = l_run[r] * corr[r] + rs[r];
-#pragma unroll
-    for (int i = 0; i < HD / 8; ++i) {
-      o[i][0] *= corr[0];
-      o[i][1] *= corr[0];
-      o[i][2] *= corr[1];
-      o[i][3] *= corr[1];
-    }
-    // ---- O += P V
-#pragma unroll
-    for (int kk2 = 0; kk2 < 4; ++kk2) {
-      uint32_t pa[4];
-      pa[0] = pack_bf16(s[2 * kk2][0], s[2 * kk2][1]);
-      pa[1] = pack_bf16(s[2 * kk2][2], s[2 * kk2][3]);
-      pa[2] = pack_bf16(s[2 * kk2 + 1][0], s[2 * kk2 + 1][1]);
-      pa[3] = pack_bf16(s[2 * kk2 + 1][2], s[2 * kk2 + 1][3]);
-#pragma unroll
-      for (int dp = 0; dp < HD / 16; ++dp) {
-        const int key = kk2 * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-        const int chunk = dp * 2 + (lane >> 4);
-        uint32_t b0, b1, b2, b3;
-        ldsm_x4_t(smem_u32(v_t + (chunk >> 3) * C::KV_HALF) + sw128(key, chunk & 7), b0, b1, b2, b3);
-        mma_bf16_16816(o[2 * dp], pa, b0, b1);
-        mma_bf16_16816(o[2 * dp + 1], pa, b2, b3);
-      }
-    }
-    __syncthreads();  // every warp is done with this buffer
-    if (threadIdx.x == 0 && j + 2 < n_tiles) issue_kv(j + 2);
   }
 
-  if (!ok) {
-    // Tiles j_fail and j_fail+1 may still be in flight: let them land before the CTA exits.
-    if (threadIdx.x == 0) {
-      mbar_wait_drain(bar_q, 0);
-      for (int j = j_fail; j < min(n_tiles, j_fail + 2); ++j) mbar_wait_drain(&bar_kv[j & 1], (j >> 1) & 1);
-    }
-    return;
-  }
-
-  // ---- normalise and store
-#pragma unroll
-  for (int r = 0; r < 2; ++r) {
-    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 1);
-    l_run[r] += __shfl_xor_sync(0xffffffffu, l_run[r], 2);
-  }
-  const float inv0 = l_run[0] > 0.f ? 1.f / l_run[0] : 0.f;
-  const float inv1 = l_run[1] > 0.f ? 1.f / l_run[1] : 0.f;
-  const int row0 = qpos0, row1 = qpos0 + 8;
-  bf16* out0 = a.out + (int64_t)(seq_start + row0) * a.ldo + head * HD;
-  bf16* out1 = a.out + (int64_t)(seq_start + row1) * a.ldo + head * HD;
-#pragma unroll
-  for (int i = 0; i < HD / 8; ++i) {
-    const int col = i * 8 + 2 * t4;
-    if (row0 < len) *reinterpret_cast<uint32_t*>(out0 + col) = pack_bf16(o[i][0] * inv0, o[i][1] * inv0);
-    if (row1 < len) *reinterpret_cast<uint32_t*>(out1 + col) = pack_bf16(o[i][2] * inv1, o[i][3] * inv1);
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
   }
 }
 
@@ -227,14 +321,14 @@ static cudaError_t launch_hd(const CUtensorMap& tmQ, const CUtensorMap& tmK, con
                              const PrefillAttnArgs& a, int n_items, cudaStream_t s) {
   static bool configured = false;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_prefill_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         PrefillCfg<HD>::SMEM);
+    cudaError_t e = cudaFuncSetAttribute(attn_prefill_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         FaCfg<HD>::SMEM);
     if (e != cudaSuccess) return e;
     configured = true;
   }
   const int64_t grid = (int64_t)n_items * a.n_q;
   if (grid == 0) return cudaSuccess;
-  attn_prefill_kernel<HD><<<(unsigned)grid, 256, PrefillCfg<HD>::SMEM, s>>>(tmQ, tmK, tmV, a);
+  attn_prefill_tc_kernel<HD><<<(unsigned)grid, 192, FaCfg<HD>::SMEM, s>>>(tmQ, tmK, tmV, a);
   return cudaGetLastError();
 }
 

@@ -234,7 +234,7 @@ __global__ void __launch_bounds__(192, 1)
     for (int tile = blockIdx.x; tile < num_tiles; tile += gridDim.x) {
       int m_blk, n_blk, split;
       gemm_tile_coords(p, tile, m_blk, n_blk, split);
-      if (!mbar_wait(&acc_full[acc], acc_phase, p.err)) break;
+      if (!__all_sync(0xffffffffu, mbar_wait(&acc_full[acc], acc_phase, p.err))) break;  // warp-uniform
       tc_fence_after();
       const int row = m_blk * C::BM + row_in_tile;
       const bool row_ok = row < p.M;

@@ -86,8 +86,9 @@ cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cu
 // ------------------------------------------------------------------ RoPE + KV write
 // One block per token.  q and k heads are rotated pairwise (i, i + hd/2) by
 // angle pos * theta^(-2i/hd) (cos/sin from the table), rounded to bf16 and
-// written to the rotated-query buffer or the key cache; v heads are copied
-// to the value cache.  Cache row of (layer, page, kv head, slot-in-page).
+// written to the rotated-query buffer or the key cache ([page][kv head][64
+// tokens][hd]); v heads are copied to the value cache, which holds each page
+// transposed ([page][kv head][hd][64 tokens]).
 __global__ void rope_kv_kernel(const RopeKvArgs a) {
   const int t = blockIdx.x;
   int slot, pos;
@@ -132,10 +133,11 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
         dst[i + half] = y1;
       }
     } else {
+      // values are stored transposed per page: [page][kv head][hd][64 keys]
       const int g = h - a.n_q - a.n_kv;
-      bf16* dst = a.v_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + g) * 64 + in_page) * a.hd;
-      dst[i] = __float2bfloat16(x0);
-      dst[i + half] = __float2bfloat16(x1);
+      bf16* dst = a.v_cache + a.layer_row0 * a.hd + (((int64_t)page * a.n_kv + g) * a.hd + i) * 64 + in_page;
+      dst[0] = __float2bfloat16(x0);
+      dst[(int64_t)half * 64] = __float2bfloat16(x1);
     }
   }
 }
@@ -360,9 +362,8 @@ __global__ void read_kv_kernel(const bf16* k_cache, const bf16* v_cache, const i
     const int t = (int)(k / ((int64_t)hd * n_kv));
     const int pos = start + t;
     const int page = block_table[(int64_t)slot * max_pages + (pos >> 6)];
-    const int64_t src = (layer_row0 + ((int64_t)page * n_kv + g) * 64 + (pos & 63)) * hd + i;
-    k_dst[k] = k_cache[src];
-    v_dst[k] = v_cache[src];
+    k_dst[k] = k_cache[(layer_row0 + ((int64_t)page * n_kv + g) * 64 + (pos & 63)) * hd + i];
+    v_dst[k] = v_cache[layer_row0 * hd + (((int64_t)page * n_kv + g) * hd + i) * 64 + (pos & 63)];
   }
 }
 cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,

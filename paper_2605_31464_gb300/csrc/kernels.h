@@ -28,7 +28,8 @@ struct PrefillAttnArgs {
   const int32_t* block_table; // [slots][max_pages]
   int max_pages;
   int n_q, n_kv;
-  int64_t layer_row0;         // first cache row of this layer: layer * num_pages * n_kv * 64
+  int64_t layer_row0;         // first K-cache row (64-token page rows of hd) of this layer
+  int64_t layer_vrow0;        // first V-cache row (rows of 64 keys, V stored transposed per page)
   bf16* out;                  // [T, n_q*hd]
   int64_t ldo;
   float scale_log2;           // log2(e) / sqrt(hd)
@@ -48,6 +49,7 @@ struct DecodeAttnArgs {
   int max_pages;
   int n_q, n_kv;
   int64_t layer_row0;
+  int64_t layer_vrow0;
   int chunk;                  // keys per split, multiple of 64
   int max_splits;
   float* part_o;              // [B][n_kv][max_splits][16][hd] unnormalised partial outputs
@@ -108,7 +110,9 @@ cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32
                            bf16* v_dst, cudaStream_t s);
 
 // Defined in runtime.cu for entry points of other translation units.
+// K cache: rows of hd, boxes {64, 64}; V cache (transposed pages): rows of 64 keys, boxes {64, hd}.
 int encode_kv_map(CUtensorMap* m, const void* base, int hd, uint64_t rows);
+int encode_vt_map(CUtensorMap* m, const void* base, int hd, uint64_t rows);
 void set_error_short(const char* msg);
 
 }  // namespace gf

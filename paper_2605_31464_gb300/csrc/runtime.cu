@@ -316,6 +316,7 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
 }
 
 int64_t layer_row0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * 64; }
+int64_t layer_vrow0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * m->hd; }
 
 
 
@@ -480,6 +481,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     pa.n_q = m->nq;
     pa.n_kv = m->nkv;
     pa.layer_row0 = layer_row0(m, l);
+    pa.layer_vrow0 = layer_vrow0(m, l);
     pa.out = m->attn;
     pa.ldo = m->q_dim;
     pa.scale_log2 = scale_log2;
@@ -568,6 +570,7 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     da.n_q = m->nq;
     da.n_kv = m->nkv;
     da.layer_row0 = layer_row0(m, l);
+    da.layer_vrow0 = layer_vrow0(m, l);
     da.chunk = m->dec_chunk;
     da.max_splits = m->dec_max_splits;
     da.part_o = m->part_o;
@@ -683,6 +686,19 @@ int encode_kv_map(CUtensorMap* m, const void* base, int hd, uint64_t rows) {
   cuuint64_t dims[2] = {(cuuint64_t)hd, rows};
   cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
   cuuint32_t box[2] = {64, 64};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS
+             ? 0
+             : 1;
+}
+int encode_vt_map(CUtensorMap* m, const void* base, int hd, uint64_t rows) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return 1;
+  cuuint64_t dims[2] = {64, rows};
+  cuuint64_t strides[1] = {128};
+  cuuint32_t box[2] = {64, (cuuint32_t)hd};
   cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -859,7 +875,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   for (int sl = m->B_max - 1; sl >= 0; --sl) m->free_slots.push_back(sl);
   const uint64_t rows = (uint64_t)m->L * m->num_pages * m->nkv * 64;
   if ((rc = make_map(&m->tm_k, m->k_cache, hd, rows, hd * 2, 64, 64))) return bail(rc);
-  if ((rc = make_map(&m->tm_v, m->v_cache, hd, rows, hd * 2, 64, 64))) return bail(rc);
+  if ((rc = make_map(&m->tm_v, m->v_cache, 64, rows / 64 * hd, 128, 64, hd))) return bail(rc);
   if ((rc = upload_block_table(m, s))) return bail(rc);
   if (cudaStreamSynchronize(s) != cudaSuccess) return bail(fail(GF_ECUDA, "create: sync failed"));
   *out = m;
@@ -1093,7 +1109,7 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
   TRY(make_map(&tk, k_cache, head_dim, rows, head_dim * 2, 64, 64));
-  TRY(make_map(&tv, v_cache, head_dim, rows, head_dim * 2, 64, 64));
+  TRY(make_map(&tv, v_cache, 64, (uint64_t)num_pages * n_kv * head_dim, 128, 64, head_dim));
   gf::DecodeAttnArgs da{};
   da.q = reinterpret_cast<const bf16*>(q);
   da.ldq = (int64_t)n_q * head_dim;
@@ -1106,6 +1122,7 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   da.n_q = n_q;
   da.n_kv = n_kv;
   da.layer_row0 = 0;
+  da.layer_vrow0 = 0;
   da.chunk = 256;
   da.max_splits = (max_ctx + 255) / 256;
   da.part_o = reinterpret_cast<float*>(workspace);

@@ -126,7 +126,8 @@ def make_paged(ctx, n_kv, hd, seed, page_order_seed=11):
         v = oracle.bf16_bits_to_f64(vbits[idx]).transpose(0, 2, 1, 3).reshape(-1, n_kv, hd)[:ctx[b]]
         dense.append((k, v))
     to = lambda x: torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).cuda()
-    return to(kbits), to(vbits), torch.from_numpy(table).cuda(), dense, max_pages
+    # the value cache holds each page transposed: [page][kv head][hd][64 tokens]
+    return to(kbits), to(vbits.transpose(0, 1, 3, 2)), torch.from_numpy(table).cuda(), dense, max_pages
 
 
 @pytest.mark.parametrize("n_q,n_kv,hd", [(28, 4, 128), (12, 2, 128), (4, 4, 64), (40, 8, 128)])

@@ -47,7 +47,7 @@ def _paged_case(ctx, n_q, n_kv, hd, seed):
         return torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).cuda()
 
     kc = bf16(1, n_pages * n_kv * 64 * hd).reshape(n_pages, n_kv, 64, hd)
-    vc = bf16(2, n_pages * n_kv * 64 * hd).reshape(n_pages, n_kv, 64, hd)
+    vc = bf16(2, n_pages * n_kv * 64 * hd).reshape(n_pages, n_kv, hd, 64)  # pages stored transposed
     q = bf16(3, B * n_q * hd).reshape(B, n_q * hd)
     return dict(q=q, kc=kc, vc=vc, table=torch.from_numpy(table).cuda(),
                 ctx=torch.tensor(ctx, dtype=torch.int32, device="cuda"), max_ctx=max(ctx), B=B, n_q=n_q, n_kv=n_kv,
