@@ -171,8 +171,8 @@ int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdic
  *          GF_GEMM_ADD_F32:    out += acc (non-atomic, as on the residual stream)
  *          GF_GEMM_ATOMIC_F32: out += acc with atomics (split-K partial sums)
  *          GF_GEMM_STORE_BF16: out (bf16) = acc
- *          GF_GEMM_SWIGLU:     W rows hold blocks of 64 gate rows followed by 64
- *                              up rows; out (bf16, N/2 columns) = silu(gate) * up
+ *          GF_GEMM_SWIGLU:     W rows hold blocks of 16 gate rows followed by the
+ *                              16 matching up rows; out (bf16, N/2 columns) = silu(gate) * up
  *   bn     tile width 64, 128 or 256, or 0 to choose; splits: split-K factor
  *          (only with GF_GEMM_ATOMIC_F32), 0 to choose; group_m: 128-row blocks
  *          per raster group (concurrent tiles share A and W tiles in L2), 0 to choose.

@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
                                                           const __grid_constant__ CUtensorMap tmV,
                                                           const DecodeAttnArgs a) {
   using C = DecodeCfg<HD>;
+  pdl_trigger();
+  pdl_wait();
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
@@ -238,6 +240,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
 // Merge the per-chunk partials of each (sequence, query head) and normalise.
 template <int HD>
 __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x / a.n_q;
   const int h = blockIdx.x % a.n_q;
   const int G = a.n_q / a.n_kv;
@@ -271,11 +275,9 @@ static cudaError_t launch_hd(const CUtensorMap& tmK, const CUtensorMap& tmV, con
   }
   if (B == 0) return cudaSuccess;
   dim3 grid(a.max_splits, a.n_kv, B);
-  attn_decode_kernel<HD><<<grid, 128, DecodeCfg<HD>::SMEM, s>>>(tmK, tmV, a);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_pdl(attn_decode_kernel<HD>, grid, dim3(128), DecodeCfg<HD>::SMEM, s, tmK, tmV, a);
   if (e != cudaSuccess) return e;
-  attn_combine_kernel<HD><<<B * a.n_q, HD, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(attn_combine_kernel<HD>, dim3(B * a.n_q), dim3(HD), 0, s, a);
 }
 
 cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a,

@@ -45,6 +45,8 @@ __global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_co
                                                                  const __grid_constant__ CUtensorMap tmV,
                                                                  const PrefillAttnArgs a) {
   using C = FaCfg<HD>;
+  pdl_trigger();
+  pdl_wait();
   constexpr uint32_t IDESC_S = idesc_bf16_f32(128, C::BKV);
   constexpr uint32_t IDESC_O = idesc_bf16_f32(128, HD);
   extern __shared__ uint8_t smem_raw[];
@@ -328,8 +330,7 @@ static cudaError_t launch_hd(const CUtensorMap& tmQ, const CUtensorMap& tmK, con
   }
   const int64_t grid = (int64_t)n_items * a.n_q;
   if (grid == 0) return cudaSuccess;
-  attn_prefill_tc_kernel<HD><<<(unsigned)grid, 192, FaCfg<HD>::SMEM, s>>>(tmQ, tmK, tmV, a);
-  return cudaGetLastError();
+  return launch_pdl(attn_prefill_tc_kernel<HD>, dim3((unsigned)grid), dim3(192), FaCfg<HD>::SMEM, s, tmQ, tmK, tmV, a);
 }
 
 cudaError_t launch_attn_prefill(int hd, const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,

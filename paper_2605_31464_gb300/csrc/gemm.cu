@@ -12,39 +12,52 @@ int gemm_smem_bytes(int bn) {
   return bn == 256 ? GemmCfg<256>::SMEM_BYTES : (bn == 128 ? GemmCfg<128>::SMEM_BYTES : GemmCfg<64>::SMEM_BYTES);
 }
 
-template <int BN, int MODE>
+template <int BN, int MODE, bool SWAP>
 static cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int grid,
                               cudaStream_t s) {
   static bool configured = false;
-  auto kern = gemm_tc_kernel<BN, MODE>;
+  auto kern = gemm_tc_kernel<BN, MODE, SWAP>;
   if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN>::SMEM_BYTES);
+    cudaError_t e =
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN, SWAP>::SMEM_BYTES);
     if (e != cudaSuccess) return e;
     configured = true;
   }
-  kern<<<grid, GemmCfg<BN>::THREADS, GemmCfg<BN>::SMEM_BYTES, s>>>(tmA, tmB, p);
-  return cudaGetLastError();
+  return launch_pdl(kern, dim3(grid), dim3(GemmCfg<BN, SWAP>::THREADS), GemmCfg<BN, SWAP>::SMEM_BYTES, s, tmA, tmB,
+                    p);
 }
 
 template <int BN>
 static cudaError_t dispatch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int mode,
                                  int grid, cudaStream_t s) {
   switch (mode) {
-    case kStoreF32: return launch_one<BN, kStoreF32>(tmA, tmB, p, grid, s);
-    case kAddF32: return launch_one<BN, kAddF32>(tmA, tmB, p, grid, s);
-    case kAtomicF32: return launch_one<BN, kAtomicF32>(tmA, tmB, p, grid, s);
-    case kStoreBF16: return launch_one<BN, kStoreBF16>(tmA, tmB, p, grid, s);
-    case kSwiGLU:
-      if (BN >= 128) return launch_one<(BN >= 128 ? BN : 128), kSwiGLU>(tmA, tmB, p, grid, s);
-      return cudaErrorInvalidValue;
+    case kStoreF32: return launch_one<BN, kStoreF32, false>(tmA, tmB, p, grid, s);
+    case kAddF32: return launch_one<BN, kAddF32, false>(tmA, tmB, p, grid, s);
+    case kAtomicF32: return launch_one<BN, kAtomicF32, false>(tmA, tmB, p, grid, s);
+    case kStoreBF16: return launch_one<BN, kStoreBF16, false>(tmA, tmB, p, grid, s);
+    case kSwiGLU: return launch_one<BN, kSwiGLU, false>(tmA, tmB, p, grid, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int BN>
+static cudaError_t dispatch_swap(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int mode,
+                                 int grid, cudaStream_t s) {
+  switch (mode) {
+    case kStoreF32: return launch_one<BN, kStoreF32, true>(tmA, tmB, p, grid, s);
+    case kAtomicF32: return launch_one<BN, kAtomicF32, true>(tmA, tmB, p, grid, s);
+    case kSwiGLU: return launch_one<BN, kSwiGLU, true>(tmA, tmB, p, grid, s);
     default: return cudaErrorInvalidValue;
   }
 }
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
-                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m) {
+                        int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
+                        bool swap) {
   if (M <= 0 || N <= 0) return cudaSuccess;
-  if (K % 64 != 0 || N % 32 != 0) return cudaErrorInvalidValue;
+  if (K % 64 != 0) return cudaErrorInvalidValue;
+  if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
+  if (swap && (M % 32 != 0 || N > bn)) return cudaErrorInvalidValue;
   GemmArgs p;
   p.M = M;
   p.N = N;
@@ -70,6 +83,14 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   const int tiles = p.num_m * p.num_n * p.splits;
   if (grid > tiles) grid = tiles;
   if (grid < 1) grid = 1;
+  if (swap) {
+    switch (bn) {
+      case 32: return dispatch_swap<32>(tmA, tmB, p, mode, grid, s);
+      case 64: return dispatch_swap<64>(tmA, tmB, p, mode, grid, s);
+      case 128: return dispatch_swap<128>(tmA, tmB, p, mode, grid, s);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (bn) {
     case 64: return dispatch_mode<64>(tmA, tmB, p, mode, grid, s);
     case 128: return dispatch_mode<128>(tmA, tmB, p, mode, grid, s);

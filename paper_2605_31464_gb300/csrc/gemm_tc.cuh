@@ -9,10 +9,17 @@
 //   kAddF32     C += acc                        (fp32 residual stream)
 //   kAtomicF32  C += acc with atomics           (split-K partial sums)
 //   kStoreBF16  C = bf16(acc)
-//   kSwiGLU     B rows are interleaved in blocks of 64 (gate, up); the
-//               output is bf16(silu(gate) * up) with N/2 columns.
+//   kSwiGLU     B rows are interleaved in blocks of 16 (16 gate rows, then
+//               the 16 matching up rows); the output is bf16(silu(gate) * up)
+//               with N/2 columns.
 // The kernel is persistent: gridDim.x CTAs walk the tile list (grouped along
 // M so that concurrently running CTAs share A and B tiles in L2).
+//
+// SWAP (decode, few activation rows): the weights are the 128-row A operand
+// and the activations the narrow B operand (N = BN >= batch rows), so each
+// pipeline stage carries mostly weight bytes; the epilogue writes the
+// transposed tile, out[b][n].  With the 16-row gate/up interleave a gate row
+// and its up row sit 16 TMEM lanes apart in the same warp.
 #pragma once
 
 #include "ptx.cuh"
@@ -31,15 +38,16 @@ struct GemmArgs {
   int* err;
 };
 
-template <int BN>
+template <int BN, bool SWAP = false>
 struct GemmCfg {
   static constexpr int BM = 128;
   static constexpr int BK = 64;
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES = BN == 256 ? 4 : (BN == 128 ? 6 : 8);
-  static constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulator buffers (128, 256 or 512 columns)
+  static constexpr int STAGES_FIT = (220 * 1024) / STAGE_BYTES;
+  static constexpr int STAGES = STAGES_FIT > 12 ? 12 : STAGES_FIT;
+  static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // two accumulator buffers
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
   static constexpr int THREADS = 192;
 };
@@ -95,11 +103,11 @@ __device__ __forceinline__ void gemm_epilogue_chunk(const GemmArgs& p, int row, 
   }
 }
 
-template <int BN, int MODE>
+template <int BN, int MODE, bool SWAP = false>
 __global__ void __launch_bounds__(192, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                    const GemmArgs p) {
-  using C = GemmCfg<BN>;
+  using C = GemmCfg<BN, SWAP>;
   constexpr uint32_t IDESC = idesc_bf16_f32(C::BM, BN);
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -140,9 +148,27 @@ __global__ void __launch_bounds__(192, 1)
   const uint32_t tmem_base = *tmem_slot;
   const int num_tiles = p.num_m * p.num_n * p.splits;
 
+  pdl_trigger();
   if (warp == 0) {
     // ------------------------------------------------ TMA producer
     if (lane == 0) {
+      // The weights (A when SWAP, else B) are never written by an earlier kernel: the weight
+      // halves of the first stages are requested before waiting for the previous kernel.
+      int pre = 0;
+      for (int tile = blockIdx.x; tile < num_tiles && pre < C::STAGES; tile += gridDim.x) {
+        int m_blk, n_blk, split;
+        gemm_tile_coords(p, tile, m_blk, n_blk, split);
+        const int kb0 = split * p.kb_per_split;
+        const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
+        for (int kb = kb0; kb < kb1 && pre < C::STAGES; ++kb, ++pre) {
+          mbar_arrive_expect_tx(&full[pre], C::STAGE_BYTES);
+          if (SWAP)
+            tma_load_2d(sA + pre * C::A_BYTES, &tmA, &full[pre], kb * C::BK, m_blk * C::BM);
+          else
+            tma_load_2d(sB + pre * C::B_BYTES, &tmB, &full[pre], kb * C::BK, n_blk * BN);
+        }
+      }
+      pdl_wait();
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
@@ -153,13 +179,21 @@ __global__ void __launch_bounds__(192, 1)
         const int kb0 = split * p.kb_per_split;
         const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
         for (int kb = kb0; kb < kb1; ++kb) {
-          if (!mbar_wait(&empty[stage], phase ^ 1u, p.err)) {
-            ok = false;
-            break;
+          if (issued < pre) {
+            // barrier armed and weight half requested above: add the activation half
+            if (SWAP)
+              tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
+            else
+              tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
+          } else {
+            if (!mbar_wait(&empty[stage], phase ^ 1u, p.err)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
+            tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
+            tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
           }
-          mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
-          tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
-          tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
           ++issued;
           if (++stage == C::STAGES) {
             stage = 0;
@@ -168,7 +202,7 @@ __global__ void __launch_bounds__(192, 1)
         }
       }
       // Every copy this thread started must have landed before the CTA exits.
-      const int outstanding = min(issued, C::STAGES);
+      const int outstanding = min(max(issued, pre), C::STAGES);
       for (int i = 0; i < outstanding; ++i) {
         if (--stage < 0) {
           stage = C::STAGES - 1;
@@ -227,6 +261,7 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else {
     // ------------------------------------------------ epilogue (warps 2..5)
+    pdl_wait();  // the epilogue writes (and may read) buffers of earlier kernels
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const int row_in_tile = quarter * 32 + lane;
     int acc = 0;
@@ -239,37 +274,61 @@ __global__ void __launch_bounds__(192, 1)
       const int row = m_blk * C::BM + row_in_tile;
       const bool row_ok = row < p.M;
       const uint32_t taddr = tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * BN);
-      if (MODE == kSwiGLU) {
+      if (SWAP) {
+        // TMEM lane = weight row (output feature), column = activation row (batch)
 #pragma unroll 1
-        for (int g = 0; g < BN / 128; ++g) {
-#pragma unroll 1
-          for (int h = 0; h < 2; ++h) {
-            uint32_t rg[32], ru[32];
-            tmem_ld32(taddr + g * 128 + h * 32, rg);
-            tmem_ld32(taddr + g * 128 + 64 + h * 32, ru);
-            tmem_ld_wait();
-            const int gate_col = n_blk * BN + g * 128 + h * 32;
-            if (row_ok && gate_col < p.N) {
-              const int out_col = n_blk * (BN / 2) + g * 64 + h * 32;
-              uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) +
-                                                    (int64_t)row * p.ldo + out_col);
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c, r);
+          tmem_ld_wait();
+          if (MODE == kSwiGLU) {
+            // lanes 0..15 of each warp hold gate rows, lanes 16..31 the matching up rows
+            const int f = m_blk * 64 + quarter * 16 + (lane & 15);
+            const bool f_ok = (lane < 16) && (f < p.M / 2);
 #pragma unroll
-              for (int i = 0; i < 4; ++i) {
-                float o[8];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  const float gv = __uint_as_float(rg[8 * i + j]);
-                  const float uv = __uint_as_float(ru[8 * i + j]);
-                  o[j] = gv / (1.0f + __expf(-gv)) * uv;
-                }
-                uint4 v;
-                v.x = pack_bf16(o[0], o[1]);
-                v.y = pack_bf16(o[2], o[3]);
-                v.z = pack_bf16(o[4], o[5]);
-                v.w = pack_bf16(o[6], o[7]);
-                dst[i] = v;
+            for (int i = 0; i < 32; ++i) {
+              const float u = __shfl_down_sync(0xffffffffu, __uint_as_float(r[i]), 16);
+              const int bb = c + i;
+              if (f_ok && bb < p.N) {
+                const float g = __uint_as_float(r[i]);
+                reinterpret_cast<__nv_bfloat16*>(p.out)[(int64_t)bb * p.ldo + f] =
+                    __float2bfloat16(g / (1.0f + __expf(-g)) * u);
               }
             }
+          } else if (row_ok) {
+            float* out = reinterpret_cast<float*>(p.out);
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int bb = c + i;
+              if (bb < p.N) {
+                if (MODE == kAtomicF32)
+                  atomicAdd(out + (int64_t)bb * p.ldo + row, __uint_as_float(r[i]));
+                else
+                  out[(int64_t)bb * p.ldo + row] = __uint_as_float(r[i]);
+              }
+            }
+          }
+        }
+      } else if (MODE == kSwiGLU) {
+        // each 32-column chunk holds 16 gate columns then the 16 matching up columns
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c, r);
+          tmem_ld_wait();
+          const int col = n_blk * BN + c;
+          if (row_ok && col < p.N) {
+            uint32_t o[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+              const float g0 = __uint_as_float(r[2 * j]), g1 = __uint_as_float(r[2 * j + 1]);
+              const float u0 = __uint_as_float(r[16 + 2 * j]), u1 = __uint_as_float(r[16 + 2 * j + 1]);
+              o[j] = pack_bf16(g0 / (1.0f + __expf(-g0)) * u0, g1 / (1.0f + __expf(-g1)) * u1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + (int64_t)row * p.ldo +
+                                                  col / 2);
+            dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+            dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
           }
         }
       } else {

@@ -10,6 +10,8 @@ namespace gf {
 // out[t, :] = float(table[ids[t], :]); an id outside [0, vocab) records
 // GF_EINVAL in the error word and yields a zero row.
 __global__ void embed_kernel(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err) {
+  pdl_trigger();
+  pdl_wait();
   const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (t >= T) return;
@@ -34,14 +36,15 @@ __global__ void embed_kernel(const int32_t* ids, int T, const bf16* table, int v
 cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err,
                          cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
-  embed_kernel<<<(T + 7) / 8, 256, 0, s>>>(ids, T, table, vocab, d, out, err);
-  return cudaGetLastError();
+  return launch_pdl(embed_kernel, dim3((T + 7) / 8), dim3(256), 0, s, ids, T, table, vocab, d, out, err);
 }
 
 // ------------------------------------------------------------------ RMSNorm
 // y[r, :] = bf16(x[src, :] * rsqrt(mean(x[src, :]^2) + eps) * gain), src = row_idx ? row_idx[r] : r.
 __global__ void rmsnorm_kernel(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d,
                                const float* gain, float eps, bf16* y, int64_t ldy) {
+  pdl_trigger();
+  pdl_wait();
   const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
@@ -69,18 +72,18 @@ __global__ void rmsnorm_kernel(const float* x, int64_t ldx, const int32_t* row_i
 cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
                            float eps, bf16* y, int64_t ldy, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  rmsnorm_kernel<<<(rows + 7) / 8, 256, 0, s>>>(x, ldx, row_idx, rows, d, gain, eps, y, ldy);
-  return cudaGetLastError();
+  return launch_pdl(rmsnorm_kernel, dim3((rows + 7) / 8), dim3(256), 0, s, x, ldx, row_idx, rows, d, gain, eps, y, ldy);
 }
 
 __global__ void last_rows_kernel(const int32_t* offsets, int B, int32_t* row_idx) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) row_idx[b] = offsets[b + 1] - 1;
 }
 cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
-  last_rows_kernel<<<(B + 255) / 256, 256, 0, s>>>(offsets, B, row_idx);
-  return cudaGetLastError();
+  return launch_pdl(last_rows_kernel, dim3((B + 255) / 256), dim3(256), 0, s, offsets, B, row_idx);
 }
 
 // ------------------------------------------------------------------ RoPE + KV write
@@ -90,6 +93,8 @@ cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cu
 // tokens][hd]); v heads are copied to the value cache, which holds each page
 // transposed ([page][kv head][hd][64 tokens]).
 __global__ void rope_kv_kernel(const RopeKvArgs a) {
+  pdl_trigger();
+  pdl_wait();
   const int t = blockIdx.x;
   int slot, pos;
   if (a.offsets) {
@@ -144,8 +149,7 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
 
 cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s) {
   if (a.T <= 0) return cudaSuccess;
-  rope_kv_kernel<<<a.T, 256, 0, s>>>(a);
-  return cudaGetLastError();
+  return launch_pdl(rope_kv_kernel, dim3(a.T), dim3(256), 0, s, a);
 }
 
 // (cos, sin) of pos * theta^(-2i/hd), evaluated in double precision.
@@ -170,6 +174,8 @@ cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cuda
 // out2[b*stride + col] with col = col_base (+ *step when step is given), if col < col_limit.
 __global__ void argmax_kernel(const float* logits, int64_t ld, int V, int32_t* out, int32_t* out2,
                               int64_t out2_stride, const int32_t* step, int col_base, int col_limit) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x;
   const float* row = logits + (int64_t)b * ld;
   float best = -INFINITY;
@@ -224,8 +230,8 @@ __global__ void argmax_kernel(const float* logits, int64_t ld, int V, int32_t* o
 cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
                           int64_t out2_stride, cudaStream_t s, const int32_t* step, int col_base, int col_limit) {
   if (B <= 0) return cudaSuccess;
-  argmax_kernel<<<B, 1024, 0, s>>>(logits, ld, V, out, out2, out2_stride, step, col_base, col_limit);
-  return cudaGetLastError();
+  return launch_pdl(argmax_kernel, dim3(B), dim3(1024), 0, s, logits, ld, V, out, out2, out2_stride, step, col_base,
+                    col_limit);
 }
 
 // ------------------------------------------------------------------ verdict (Sec. 2.1)
@@ -235,6 +241,8 @@ struct VerdictIds {
 };
 __global__ void verdict_kernel(const float* logits, int64_t ld, int B, VerdictIds ids, int K, float tau, float* p,
                                float* conf, int32_t* arg, uint8_t* defer) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= B) return;
   const float* row = logits + (int64_t)b * ld;
@@ -268,38 +276,42 @@ cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t
   if (B <= 0) return cudaSuccess;
   VerdictIds v;
   for (int k = 0; k < 8; ++k) v.v[k] = k < K ? ids[k] : 0;
-  verdict_kernel<<<(B + 127) / 128, 128, 0, s>>>(logits, ld, B, v, K, tau, p, conf, arg, defer);
-  return cudaGetLastError();
+  return launch_pdl(verdict_kernel, dim3((B + 127) / 128), dim3(128), 0, s, logits, ld, B, v, K, tau, p, conf, arg,
+                    defer);
 }
 
 // ------------------------------------------------------------------ bookkeeping
 __global__ void set_seq_len_kernel(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) seq_len[slots[b]] = offsets[b + 1] - offsets[b];
 }
 cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
                                cudaStream_t s) {
   if (B <= 0) return cudaSuccess;
-  set_seq_len_kernel<<<(B + 255) / 256, 256, 0, s>>>(offsets, slots, B, seq_len);
-  return cudaGetLastError();
+  return launch_pdl(set_seq_len_kernel, dim3((B + 255) / 256), dim3(256), 0, s, offsets, slots, B, seq_len);
 }
 
 // seq_len[handles[b]] += 1 for every b; *step += 1 when step is given (decode-step counter).
 __global__ void advance_kernel(const int32_t* handles, int B, int32_t* seq_len, int32_t* step) {
+  pdl_trigger();
+  pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b < B) seq_len[handles[b]] += 1;
   if (step && b == 0) *step += 1;
 }
 cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s, int32_t* step) {
   if (B <= 0) return cudaSuccess;
-  advance_kernel<<<(B + 255) / 256, 256, 0, s>>>(handles, B, seq_len, step);
-  return cudaGetLastError();
+  return launch_pdl(advance_kernel, dim3((B + 255) / 256), dim3(256), 0, s, handles, B, seq_len, step);
 }
 
 // prompt_b = inc_ids[inc_off[b]:inc_off[b+1]] ++ cand_ids[cand_off[b]:cand_off[b+1]], packed at prompt_off[b].
 __global__ void build_prompts_kernel(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                      const int32_t* cand_off, const int32_t* prompt_off, int B, int T,
                                      int32_t* out) {
+  pdl_trigger();
+  pdl_wait();
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x) {
     int lo = 0, hi = B - 1;
     while (lo < hi) {
@@ -317,21 +329,21 @@ cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off,
   if (T <= 0) return cudaSuccess;
   int blocks = (T + 255) / 256;
   if (blocks > 4096) blocks = 4096;
-  build_prompts_kernel<<<blocks, 256, 0, s>>>(inc_ids, inc_off, cand_ids, cand_off, prompt_off, B, T, out);
-  return cudaGetLastError();
+  return launch_pdl(build_prompts_kernel, dim3(blocks), dim3(256), 0, s, inc_ids, inc_off, cand_ids, cand_off,
+                    prompt_off, B, T, out);
 }
 
 // ------------------------------------------------------------------ weight packing
-// dst rows [128c, 128c+64) = gate rows [64c, 64c+64), dst rows [128c+64, 128c+128) = up rows;
+// dst rows [32c, 32c+16) = gate rows [16c, 16c+16), dst rows [32c+16, 32c+32) = up rows;
 // rows past F are zero.  Fp = F rounded up to 64.
 __global__ void pack_gate_up_kernel(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst) {
   const int64_t chunks_per_row = d / 8;
   const int64_t n = (int64_t)2 * Fp * chunks_per_row;
   for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x) {
     const int64_t r = k / chunks_per_row, c = k % chunks_per_row;
-    const int64_t blk = r / 128, in = r % 128;
-    const bool is_up = in >= 64;
-    const int64_t f = blk * 64 + (in & 63);
+    const int64_t blk = r / 32, in = r % 32;
+    const bool is_up = in >= 16;
+    const int64_t f = blk * 16 + (in & 15);
     uint4 v = make_uint4(0, 0, 0, 0);
     if (f < F) v = *reinterpret_cast<const uint4*>((is_up ? up : gate) + f * d + c * 8);
     *reinterpret_cast<uint4*>(dst + r * d + c * 8) = v;

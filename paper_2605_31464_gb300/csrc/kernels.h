@@ -10,15 +10,37 @@ namespace gf {
 
 using bf16 = __nv_bfloat16;
 
+// Launch with programmatic stream serialization: the kernel may begin while the
+// previous kernel of the stream finishes; it must call pdl_wait() (ptx.cuh)
+// before using that kernel's results.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                              Args&&... args) {
+  cudaLaunchConfig_t cfg{};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
 // ------------------------------------------------------------------ GEMM
 // C[M,N] (op)= A[M,K] . B[N,K]^T ; mode is a GemmMode.  tmA/tmB are 2D
 // tensor maps (bf16, 128-byte swizzle) with boxes {64, 128} and {64, bn}.
 int gemm_num_stages(int bn);
 int gemm_smem_bytes(int bn);
 // group_m: M-blocks per raster group (0 = sized so a group's A tiles fill about 48 MiB of L2).
+// swap: A holds the weights (M = output features, multiple of 32), B the activations
+// (N = rows <= bn, bn 32/64/128), and out is written transposed (out[n][m]); modes
+// kStoreF32, kAtomicF32 and kSwiGLU only.
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
-                        int group_m = 0);
+                        int group_m = 0, bool swap = false);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {

@@ -273,10 +273,25 @@ struct ProfScope {
   }
 };
 
-// Tile width and split-K factor for a GEMM of M rows.
-void plan_gemm(const gf_model* m, int M, int N, int K, int mode, int* bn, int* splits) {
+// Tile width, split-K factor and operand order for a GEMM of M rows.  Few rows
+// (decode) swap the operands: the weights fill the 128-row MMA dimension and the
+// rows become a narrow N, so the pipeline streams mostly weight bytes.
+void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, bool* swap) {
   const int num_m = (M + 127) / 128;
   *splits = 1;
+  *swap = false;
+  if (M <= 128 && N % 32 == 0 && (mode == gf::kStoreF32 || mode == gf::kAtomicF32 || mode == gf::kSwiGLU)) {
+    *swap = true;
+    *bn = M <= 32 ? 32 : (M <= 64 ? 64 : 128);
+    if (mode == gf::kAtomicF32) {
+      const int tiles = (N + 127) / 128;
+      const int kb = K / 64;
+      int s = (2 * sms + tiles - 1) / tiles;
+      s = std::min(s, std::max(1, kb / 4));
+      *splits = std::max(1, s);
+    }
+    return;
+  }
   if (mode == gf::kSwiGLU) {
     *bn = num_m >= 4 ? 256 : 128;
     return;
@@ -292,7 +307,7 @@ void plan_gemm(const gf_model* m, int M, int N, int K, int mode, int* bn, int* s
   *bn = 64;
   const int tiles = num_m * ((N + 63) / 64);
   const int kb = K / 64;
-  int s = (2 * m->sms + tiles - 1) / tiles;
+  int s = (2 * sms + tiles - 1) / tiles;
   s = std::min(s, std::max(1, kb / 4));
   *splits = std::max(1, s);
 }
@@ -302,15 +317,24 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
          cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0) {
   if (M <= 0) return GF_OK;
   int bn, splits;
-  plan_gemm(m, M, N, K, mode, &bn, &splits);
+  bool swap;
+  plan_gemm(m->sms, M, N, K, mode, &bn, &splits, &swap);
   CUtensorMap ta, tb;
-  TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, 128, &ta));
-  TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, (uint32_t)bn, &tb));
+  if (swap) {
+    TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, 128, &ta));
+    TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, (uint32_t)bn, &tb));
+  } else {
+    TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, 128, &ta));
+    TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, (uint32_t)bn, &tb));
+  }
   const double na = n_alg ? n_alg : N, ka = k_alg ? k_alg : K;
   const double out_bytes = (mode == gf::kSwiGLU ? na / 2 * 2 : na * (mode == gf::kStoreBF16 ? 2 : 4)) * M;
   ProfScope ps(m, s, decode ? GF_PROF_DECODE_GEMM : GF_PROF_PREFILL_GEMM, 2.0 * M * na * ka,
                na * ka * 2 + (double)M * ka * 2 + out_bytes * (mode == gf::kAddF32 || mode == gf::kAtomicF32 ? 2 : 1));
-  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
+  if (swap)
+    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true));
+  else
+    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
   m->launches += 1;
   return GF_OK;
 }
@@ -1047,9 +1071,8 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   if (!A || !W || !out || M < 0 || N < 1 || K < 64) return fail(GF_EINVAL, "bad GEMM arguments");
   if (K % 64 || N % 32) return fail(GF_EINVAL, "GEMM needs K %% 64 == 0 and N %% 32 == 0");
   if (mode < GF_GEMM_STORE_F32 || mode > GF_GEMM_SWIGLU) return fail(GF_EINVAL, "bad GEMM mode");
-  if (mode == GF_GEMM_SWIGLU && N % 128) return fail(GF_EINVAL, "SwiGLU GEMM needs N %% 128 == 0");
+  if (mode == GF_GEMM_SWIGLU && N % 32) return fail(GF_EINVAL, "SwiGLU GEMM needs N %% 32 == 0");
   if (bn != 0 && bn != 64 && bn != 128 && bn != 256) return fail(GF_EINVAL, "bn must be 0, 64, 128 or 256");
-  if (mode == GF_GEMM_SWIGLU && bn == 64) return fail(GF_EINVAL, "SwiGLU GEMM needs bn >= 128");
   if (splits > 1 && mode != GF_GEMM_ATOMIC_F32) return fail(GF_EINVAL, "split-K needs the atomic mode");
   if (ldo < (mode == GF_GEMM_SWIGLU ? N / 2 : N)) return fail(GF_EINVAL, "ldo too small");
   if (M == 0) return GF_OK;
@@ -1061,16 +1084,23 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   int dev = 0, sms = 0;
   CU(cudaGetDevice(&dev));
   CU(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
-  gf_model fake;
-  fake.sms = sms;
   int pbn, psplits;
-  plan_gemm(&fake, M, N, K, mode, &pbn, &psplits);
-  if (bn == 0) bn = pbn;
-  if (splits <= 0) splits = psplits;
+  bool swap = false;
+  plan_gemm(sms, M, N, K, mode, &pbn, &psplits, &swap);
+  const bool bn_given = bn != 0;
+  if (bn_given) swap = false;  // an explicit tile width asks for the row-major tiling
+  if (!bn_given) bn = pbn;
+  if (splits <= 0) splits = bn_given ? 1 : psplits;
   CUtensorMap ta, tb;
-  TRY(make_map(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, 128));
-  TRY(make_map(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, (uint32_t)bn));
-  CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m));
+  if (swap) {
+    TRY(make_map(&ta, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, 128));
+    TRY(make_map(&tb, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, (uint32_t)bn));
+    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m, true));
+  } else {
+    TRY(make_map(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, 128));
+    TRY(make_map(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, (uint32_t)bn));
+    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m));
+  }
   return GF_OK;
 }
 

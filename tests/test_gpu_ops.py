@@ -80,17 +80,43 @@ def test_gemm_residual_add_and_bf16_store():
 @pytest.mark.parametrize("bn", [128, 256])
 def test_gemm_swiglu_epilogue(bn):
     import paper_2605_31464_gb300 as gf
-    M, F, K = 260, 192, 320  # F = 3 blocks of 64
+    M, F, K = 260, 208, 320  # F = 13 blocks of 16
     A, a64 = _bf16((M, K), 7)
     G, g64 = _bf16((F, K), 8, 0.05)
     U, u64 = _bf16((F, K), 9, 0.05)
-    # interleave blocks of 64 rows: gate block c, then up block c
-    Wi = torch.cat([torch.cat([G[64 * c:64 * c + 64], U[64 * c:64 * c + 64]]) for c in range(F // 64)])
+    # interleave blocks of 16 rows: gate block c, then up block c
+    Wi = torch.cat([torch.cat([G[16 * c:16 * c + 16], U[16 * c:16 * c + 16]]) for c in range(F // 16)])
     out = torch.zeros(M, F, device="cuda", dtype=torch.bfloat16)
     gf.gemm(A, Wi, out, gf.GF_GEMM_SWIGLU, bn=bn)
     g = a64 @ g64.T
     ref = oracle.silu(g) * (a64 @ u64.T)
     np.testing.assert_allclose(out.float().cpu().numpy(), ref, rtol=1e-2, atol=1e-2 * np.abs(ref).max())
+
+
+@pytest.mark.parametrize("M", [1, 7, 32, 33, 100, 128])
+@pytest.mark.parametrize("mode", ["f32", "atomic", "swiglu"])
+def test_gemm_few_rows_swapped_operands(M, mode):
+    # with few rows (decode) the library puts the weights in the 128-row MMA operand
+    import paper_2605_31464_gb300 as gf
+    N, K = (4608 if mode != "swiglu" else 1024), 1024
+    A, a64 = _bf16((M, K), 11)
+    W, w64 = _bf16((N, K), 12, 0.05)
+    if mode == "swiglu":
+        out = torch.zeros(M, N // 2, device="cuda", dtype=torch.bfloat16)
+        gf.gemm(A, W, out, gf.GF_GEMM_SWIGLU)
+        gu = a64 @ w64.T
+        g = np.concatenate([gu[:, 32 * c:32 * c + 16] for c in range(N // 32)], axis=1)
+        u = np.concatenate([gu[:, 32 * c + 16:32 * c + 32] for c in range(N // 32)], axis=1)
+        ref = oracle.silu(g) * u
+        got = out.float().cpu().numpy()
+        np.testing.assert_allclose(got, ref, rtol=1e-2, atol=1e-2 * np.abs(ref).max())
+        return
+    base = torch.randn(M, N, device="cuda") if mode == "atomic" else torch.zeros(M, N, device="cuda")
+    out = base.clone()
+    gf.gemm(A, W, out, gf.GF_GEMM_ATOMIC_F32 if mode == "atomic" else gf.GF_GEMM_STORE_F32)
+    gf.gf_gemm_status(torch.cuda.current_stream().cuda_stream)
+    ref = base.cpu().double().numpy() + a64 @ w64.T
+    np.testing.assert_allclose(out.cpu().numpy(), ref, rtol=1e-4, atol=1e-4 * np.abs(ref).max())
 
 
 def test_gemm_rejects_bad_shapes():
