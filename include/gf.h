@@ -240,13 +240,16 @@ int gf_decode_attention_static(const void* q, const void* k_cache, const void* v
  * Kernel classes whose launches can be bracketed by CUDA events (on the
  * launching stream) for live timing inside a run. */
 enum { GF_PROF_PREFILL_GEMM = 0, GF_PROF_DECODE_GEMM = 1, GF_PROF_PREFILL_ATTN = 2, GF_PROF_DECODE_ATTN = 3,
-       GF_PROF_KINDS = 4 };
+       GF_PROF_DECODE_STEPS = 4, /* the replayed decode steps of gf_forecast_batch, as one interval */
+       GF_PROF_KINDS = 5 };
 /* Time every launch of the classes whose bit is set in `mask` (0 = off). */
 int gf_profile_enable(gf_model* m, uint32_t mask);
 /* Synchronise the device and return, for class `kind` since the last read:
  * launches, summed kernel milliseconds, algorithmic FLOPs (2*M*N*K for a
  * GEMM, 4*hd per visible query-key pair for attention) and algorithmic HBM
- * bytes (operands read once, outputs written once); then reset the class. */
+ * bytes (operands read once, outputs written once; for GF_PROF_DECODE_STEPS
+ * every weight once per step plus the cached keys and values each step reads
+ * and writes); then reset the class. */
 int gf_profile_read(gf_model* m, int32_t kind, int64_t* launches, double* ms, double* flops, double* bytes);
 
 /* ---- inspection hooks (parity tests at full size) -------------------------

@@ -16,14 +16,19 @@
 
 namespace gf {
 
+#ifndef GF_DECODE_STAGES
+#define GF_DECODE_STAGES 2
+#endif
+
 template <int HD>
 struct DecodeCfg {
+  static constexpr int STAGES = GF_DECODE_STAGES;   // pages (K + V^T) in flight per CTA
   static constexpr int HALVES = HD / 64;
   static constexpr int PAGE_HALF = 64 * 128;        // one 64-column half of a K page
   static constexpr int PAGE_BYTES = 64 * HD * 2;    // one page of K (or V^T) for one head
   static constexpr int Q_BYTES = 16 * HD * 2;
-  // smem: Q [HALVES][16][128 B] | K[2] | V[2] | barriers ; the K/V area is reused to combine warps
-  static constexpr int SMEM = 1024 + Q_BYTES + 4 * PAGE_BYTES + 64;
+  // smem: Q [HALVES][16][128 B] | K[STAGES] | V[STAGES] | barriers; the K/V area is reused to combine warps
+  static constexpr int SMEM = 1024 + Q_BYTES + 2 * STAGES * PAGE_BYTES + 8 * STAGES;
 };
 
 template <int HD>
@@ -37,8 +42,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* sQ = smem;
   uint8_t* sK = sQ + C::Q_BYTES;
-  uint8_t* sV = sK + 2 * C::PAGE_BYTES;
-  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + 2 * C::PAGE_BYTES);  // [2]
+  uint8_t* sV = sK + C::STAGES * C::PAGE_BYTES;
+  uint64_t* bar = reinterpret_cast<uint64_t*>(sV + C::STAGES * C::PAGE_BYTES);  // [STAGES]
 
   const int split = blockIdx.x;
   const int kvh = blockIdx.y;
@@ -56,7 +61,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int32_t* pages = a.block_table + (int64_t)slot * a.max_pages;
 
   auto issue = [&](int i) {
-    const int buf = i & 1;
+    const int buf = i % C::STAGES;
     const int64_t pg = (int64_t)pages[p0 + i] * a.n_kv + kvh;
     mbar_arrive_expect_tx(&bar[buf], 2 * C::PAGE_BYTES);
 #pragma unroll
@@ -66,12 +71,10 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   };
 
   if (threadIdx.x == 0) {
-    mbar_init(&bar[0], 1);
-    mbar_init(&bar[1], 1);
+    for (int i = 0; i < C::STAGES; ++i) mbar_init(&bar[i], 1);
     fence_mbar_init();
     fence_async_smem();
-    issue(0);
-    if (n_pages > 1) issue(1);
+    for (int i = 0; i < C::STAGES && i < n_pages; ++i) issue(i);
   }
   // Q rows of this group (zero rows beyond G), 16-byte chunks, swizzled like TMA.
   for (int c = threadIdx.x; c < 16 * (HD / 8); c += blockDim.x) {
@@ -103,8 +106,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   int i_fail = 0;
 
   for (int i = 0; i < n_pages; ++i) {
-    const int buf = i & 1;
-    if (!mbar_wait(&bar[buf], (i >> 1) & 1, a.err)) {
+    const int buf = i % C::STAGES;
+    if (!mbar_wait(&bar[buf], (i / C::STAGES) & 1, a.err)) {
       ok = false;
       i_fail = i;
       break;
@@ -182,12 +185,13 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
       mma_bf16_16816(o[2 * dp + 1], pa, b2, b3);
     }
     __syncthreads();
-    if (threadIdx.x == 0 && i + 2 < n_pages) issue(i + 2);
+    if (threadIdx.x == 0 && i + C::STAGES < n_pages) issue(i + C::STAGES);
   }
 
   if (!ok) {
     if (threadIdx.x == 0)
-      for (int i = i_fail; i < min(n_pages, i_fail + 2); ++i) mbar_wait_drain(&bar[i & 1], (i >> 1) & 1);
+      for (int i = i_fail; i < min(n_pages, i_fail + C::STAGES); ++i)
+        mbar_wait_drain(&bar[i % C::STAGES], (i / C::STAGES) & 1);
     return;
   }
 

@@ -53,7 +53,7 @@ static cudaError_t dispatch_swap(const CUtensorMap& tmA, const CUtensorMap& tmB,
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
-                        bool swap) {
+                        bool swap, unsigned long long* argmax_keys) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0) return cudaErrorInvalidValue;
   if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
@@ -80,6 +80,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   p.out = out;
   p.ldo = ldo;
   p.err = err;
+  p.argmax_keys = (swap && mode == kStoreF32) ? argmax_keys : nullptr;
   const int tiles = p.num_m * p.num_n * p.splits;
   if (grid > tiles) grid = tiles;
   if (grid < 1) grid = 1;

@@ -36,7 +36,17 @@ struct GemmArgs {
   void* out;
   int64_t ldo;  // elements
   int* err;
+  // SWAP + kStoreF32 only: per output row b, atomicMax of argmax_key(value, column) over the tile
+  // (the greedy arg max of a logits row; the lowest column wins ties)
+  unsigned long long* argmax_keys;
 };
+
+// Orders (value, index) pairs by value, then by lower index: larger key = better.
+__device__ __forceinline__ unsigned long long argmax_key(float v, int idx) {
+  const uint32_t u = __float_as_uint(v);
+  const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  return ((unsigned long long)ord << 32) | (0xFFFFFFFFu - (uint32_t)idx);
+}
 
 template <int BN, bool SWAP = false>
 struct GemmCfg {
@@ -295,17 +305,39 @@ __global__ void __launch_bounds__(192, 1)
                     __float2bfloat16(g / (1.0f + __expf(-g)) * u);
               }
             }
-          } else if (row_ok) {
+          } else {
             float* out = reinterpret_cast<float*>(p.out);
+            if (row_ok) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const int bb = c + i;
-              if (bb < p.N) {
-                if (MODE == kAtomicF32)
-                  atomicAdd(out + (int64_t)bb * p.ldo + row, __uint_as_float(r[i]));
-                else
-                  out[(int64_t)bb * p.ldo + row] = __uint_as_float(r[i]);
+              for (int i = 0; i < 32; ++i) {
+                const int bb = c + i;
+                if (bb < p.N) {
+                  if (MODE == kAtomicF32)
+                    atomicAdd(out + (int64_t)bb * p.ldo + row, __uint_as_float(r[i]));
+                  else
+                    out[(int64_t)bb * p.ldo + row] = __uint_as_float(r[i]);
+                }
               }
+            }
+            if (MODE == kStoreF32 && p.argmax_keys) {
+              // transpose-reduce the warp's 32 rows x 32 columns: after five halvings lane l holds
+              // the best key of column c + l over this warp's rows
+              unsigned long long k[32];
+#pragma unroll
+              for (int i = 0; i < 32; ++i) k[i] = row_ok ? argmax_key(__uint_as_float(r[i]), row) : 0ull;
+#pragma unroll
+              for (int o = 16; o >= 1; o >>= 1) {
+                const bool upper = (lane & o) != 0;
+#pragma unroll
+                for (int j = 0; j < o; ++j) {
+                  const unsigned long long send = upper ? k[j] : k[j + o];
+                  const unsigned long long keep = upper ? k[j + o] : k[j];
+                  const unsigned long long got = __shfl_xor_sync(0xffffffffu, send, o);
+                  k[j] = keep > got ? keep : got;
+                }
+              }
+              const int bb = c + lane;
+              if (bb < p.N && k[0] != 0ull) atomicMax(p.argmax_keys + bb, k[0]);
             }
           }
         }

@@ -306,6 +306,35 @@ cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cuda
   return launch_pdl(advance_kernel, dim3((B + 255) / 256), dim3(256), 0, s, handles, B, seq_len, step);
 }
 
+__global__ void finish_step_kernel(unsigned long long* keys, int B, int32_t* next, int32_t* tok, int64_t tok_stride,
+                                   int32_t* step, int col_base, int col_limit, const int32_t* handles,
+                                   int32_t* seq_len) {
+  pdl_trigger();
+  pdl_wait();
+  const int s = step ? *step : 0;
+  __syncthreads();
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    const unsigned long long k = keys[b];
+    keys[b] = 0ull;
+    const int id = k ? (int)(0xFFFFFFFFu - (uint32_t)(k & 0xFFFFFFFFull)) : 0;
+    next[b] = id;
+    if (tok) {
+      const int col = col_base + s;
+      if (col < col_limit) tok[(int64_t)b * tok_stride + col] = id;
+    }
+    if (seq_len) seq_len[handles[b]] += 1;
+  }
+  __syncthreads();
+  if (seq_len && step && threadIdx.x == 0) *step = s + 1;
+}
+cudaError_t launch_finish_step(unsigned long long* keys, int B, int32_t* next, int32_t* tok, int64_t tok_stride,
+                               int32_t* step, int col_base, int col_limit, const int32_t* handles,
+                               int32_t* seq_len, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  return launch_pdl(finish_step_kernel, dim3(1), dim3(1024), 0, s, keys, B, next, tok, tok_stride, step, col_base,
+                    col_limit, handles, seq_len);
+}
+
 // prompt_b = inc_ids[inc_off[b]:inc_off[b+1]] ++ cand_ids[cand_off[b]:cand_off[b+1]], packed at prompt_off[b].
 __global__ void build_prompts_kernel(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                      const int32_t* cand_off, const int32_t* prompt_off, int B, int T,

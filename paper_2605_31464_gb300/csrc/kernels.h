@@ -38,9 +38,11 @@ int gemm_smem_bytes(int bn);
 // swap: A holds the weights (M = output features, multiple of 32), B the activations
 // (N = rows <= bn, bn 32/64/128), and out is written transposed (out[n][m]); modes
 // kStoreF32, kAtomicF32 and kSwiGLU only.
+// argmax_keys (swap + kStoreF32 only): atomicMax per output row of the packed (value, column)
+// key of its largest element (see gemm_tc.cuh); the array must start at zero.
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
-                        int group_m = 0, bool swap = false);
+                        int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {
@@ -121,6 +123,12 @@ cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int
                                cudaStream_t s);
 cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s,
                            int32_t* step = nullptr);
+// Greedy tokens from the argmax keys of the LM-head GEMM: next[b] (and tok[b*stride + col],
+// col = col_base (+ *step), when col < col_limit); resets the keys; with seq_len, advances
+// seq_len[handles[b]] and then *step.  B <= 1024.
+cudaError_t launch_finish_step(unsigned long long* keys, int B, int32_t* next, int32_t* tok, int64_t tok_stride,
+                               int32_t* step, int col_base, int col_limit, const int32_t* handles,
+                               int32_t* seq_len, cudaStream_t s);
 cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                  const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
                                  cudaStream_t s);

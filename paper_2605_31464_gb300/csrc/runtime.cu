@@ -205,10 +205,12 @@ struct gf_model {
   int32_t* tok_hist = nullptr;
   int tok_stride = 0;
   int32_t* ctl = nullptr;  // [0]: device decode-step counter
+  unsigned long long* keys = nullptr;  // [B_max] fused greedy arg max keys (kept at zero between uses)
   // one CUDA graph per batch size for the decode step of gf_forecast_batch
   cudaStream_t cap_stream = nullptr;
   std::map<int, cudaGraphExec_t> graphs;
   int64_t graph_launches_per_step = 0;
+  double weight_bytes = 0;  // bytes of all linear weights and the LM head (read once per decode step)
 };
 
 namespace {
@@ -284,9 +286,10 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
     *swap = true;
     *bn = M <= 32 ? 32 : (M <= 64 ? 64 : 128);
     if (mode == gf::kAtomicF32) {
+      // about one wave of (tile, split) units: more splits add atomic traffic without adding bandwidth
       const int tiles = (N + 127) / 128;
       const int kb = K / 64;
-      int s = (2 * sms + tiles - 1) / tiles;
+      int s = (sms + tiles / 2) / tiles;
       s = std::min(s, std::max(1, kb / 4));
       *splits = std::max(1, s);
     }
@@ -313,8 +316,10 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
 }
 
 // n_alg / k_alg: the unpadded output width and contraction length (algorithmic work).
+// keys: ask the LM-head GEMM to fuse the greedy arg max (*fused tells whether it could).
 int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
-         cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0) {
+         cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0, unsigned long long* keys = nullptr,
+         bool* fused = nullptr) {
   if (M <= 0) return GF_OK;
   int bn, splits;
   bool swap;
@@ -331,8 +336,11 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
   const double out_bytes = (mode == gf::kSwiGLU ? na / 2 * 2 : na * (mode == gf::kStoreBF16 ? 2 : 4)) * M;
   ProfScope ps(m, s, decode ? GF_PROF_DECODE_GEMM : GF_PROF_PREFILL_GEMM, 2.0 * M * na * ka,
                na * ka * 2 + (double)M * ka * 2 + out_bytes * (mode == gf::kAddF32 || mode == gf::kAtomicF32 ? 2 : 1));
+  const bool use_keys = keys && swap && mode == gf::kStoreF32;
+  if (fused) *fused = use_keys;
   if (swap)
-    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true));
+    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true,
+                       use_keys ? keys : nullptr));
   else
     CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
   m->launches += 1;
@@ -340,6 +348,14 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
 }
 
 int64_t layer_row0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * 64; }
+
+// Keys per decode-attention CTA: the largest of 1024/512/256 that still gives two CTAs per SM
+// (longer chunks keep each CTA's page pipeline full and leave fewer partial results to merge).
+int decode_chunk(int B, int n_kv, int max_ctx, int sms) {
+  for (int chunk = 1024; chunk > 256; chunk /= 2)
+    if ((int64_t)B * n_kv * ((max_ctx + chunk - 1) / chunk) >= 2 * sms) return chunk;
+  return 256;
+}
 int64_t layer_vrow0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * m->hd; }
 
 
@@ -533,9 +549,15 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   CU(gf::launch_rmsnorm(m->resid, m->d, m->last_idx, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
   m->launches += 2;
   float* lg = logits_dst ? logits_dst : m->logits;
-  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, false));
+  bool fused = false;
+  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, false, 0, 0,
+           next_dst ? m->keys : nullptr, &fused));
   if (next_dst) {
-    CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+    if (fused)
+      CU(gf::launch_finish_step(m->keys, B, next_dst, tokens_col, tokens_stride, nullptr, 0, 1 << 30, nullptr,
+                                nullptr, s));
+    else
+      CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
     m->launches++;
   }
   CU(gf::launch_set_seq_len(d_off, d_slots, B, m->seq_len, s));
@@ -595,8 +617,8 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     da.n_kv = m->nkv;
     da.layer_row0 = layer_row0(m, l);
     da.layer_vrow0 = layer_vrow0(m, l);
-    da.chunk = m->dec_chunk;
-    da.max_splits = m->dec_max_splits;
+    da.chunk = decode_chunk(B, m->nkv, m->cfg.max_seq, m->sms);
+    da.max_splits = (m->dec_max_splits * m->dec_chunk + da.chunk - 1) / da.chunk;
     da.part_o = m->part_o;
     da.part_ml = m->part_ml;
     da.out = m->dattn;
@@ -621,17 +643,26 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
   CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
   m->launches++;
   float* lg = logits_dst ? logits_dst : m->logits;
-  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, true));
-  if (next_dst) {
-    if (step)
-      CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s, step, 1,
-                           (int)tokens_stride));
-    else
-      CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+  bool fused = false;
+  TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, true, 0, 0,
+           next_dst ? m->keys : nullptr, &fused));
+  if (next_dst && fused) {
+    // greedy tokens from the LM head's fused arg max; advances the sequences and the step counter
+    CU(gf::launch_finish_step(m->keys, B, next_dst, tokens_col, tokens_stride, step, step ? 1 : 0,
+                              step ? (int)tokens_stride : (1 << 30), m->handles, m->seq_len, s));
+    m->launches++;
+  } else {
+    if (next_dst) {
+      if (step)
+        CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s, step, 1,
+                             (int)tokens_stride));
+      else
+        CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
+      m->launches++;
+    }
+    CU(gf::launch_advance(m->handles, B, m->seq_len, s, step));
     m->launches++;
   }
-  CU(gf::launch_advance(m->handles, B, m->seq_len, s, step));
-  m->launches++;
   if (!capturing)
     for (int b = 0; b < B; ++b) m->h_len[h[b]] += 1;
   return GF_OK;
@@ -853,6 +884,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   m->tok_stride = c.max_seq;
   if (!rc) rc = dalloc(m, &m->tok_hist, Bm * m->tok_stride);
   if (!rc) rc = dalloc(m, &m->ctl, 4);
+  if (!rc) rc = dalloc(m, &m->keys, Bm);
   if (rc) return bail(rc);
 
   // ---- pack weights
@@ -880,6 +912,8 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
     if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->attn_norm[l]), d, W.attn_norm, s);
     if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->ffn_norm[l]), d, W.ffn_norm, s);
   }
+  m->weight_bytes = (double)m->L * ((double)m->qkv_dim * d + (double)d * m->q_dim + 2.0 * m->ffn * d +
+                                    (double)d * m->ffn) * 2 + (double)m->vocab * d * 2;
   if (e == cudaSuccess) e = cp(m->embed, w->embed, (size_t)m->vocab * d * 2);
   if (e == cudaSuccess) e = cp(m->head, w->lm_head, (size_t)m->vocab * d * 2);
   if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->final_norm), d, m->final_norm, s);
@@ -887,6 +921,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (e == cudaSuccess) e = cudaMemsetAsync(m->dqkv, 0, Bm * m->qkv_dim * sizeof(float), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(m->err, 0, sizeof(int), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(m->seq_len, 0, Bm * sizeof(int32_t), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(m->keys, 0, Bm * sizeof(unsigned long long), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return bail(fail(GF_ECUDA, "weight packing failed: %s", cudaGetErrorString(e)));
 
@@ -989,10 +1024,24 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
     if (rc == GF_OK && n_decode > 1) {
       cudaGraphExec_t exec = nullptr;
       rc = decode_graph(m, B, h.data(), &exec);
-      for (int step = 1; step < n_decode && rc == GF_OK; ++step) {
-        const cudaError_t e = cudaGraphLaunch(exec, s);
-        if (e != cudaSuccess) rc = fail(GF_ECUDA, "graph launch failed: %s", cudaGetErrorString(e));
-        m->launches += m->graph_launches_per_step;
+      // algorithmic bytes of the replayed steps: every weight once per step, the cached K/V each
+      // sequence reads, and the new K/V rows written
+      double bytes = 0;
+      if (m->prof_mask & (1u << GF_PROF_DECODE_STEPS)) {
+        const double kv_tok = (double)m->L * m->nkv * m->hd * 2 * 2;
+        for (int step = 1; step < n_decode; ++step) {
+          double ctx = 0;
+          for (int b = 0; b < B; ++b) ctx += m->h_len[h[b]] + step;  // context of this step's query
+          bytes += m->weight_bytes + ctx * kv_tok + (double)B * kv_tok;
+        }
+      }
+      {
+        ProfScope ps(m, s, GF_PROF_DECODE_STEPS, 0.0, bytes);
+        for (int step = 1; step < n_decode && rc == GF_OK; ++step) {
+          const cudaError_t e = cudaGraphLaunch(exec, s);
+          if (e != cudaSuccess) rc = fail(GF_ECUDA, "graph launch failed: %s", cudaGetErrorString(e));
+          m->launches += m->graph_launches_per_step;
+        }
       }
       if (rc == GF_OK)
         for (int b = 0; b < B; ++b) m->h_len[h[b]] += n_decode - 1;
@@ -1153,8 +1202,11 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   da.n_kv = n_kv;
   da.layer_row0 = 0;
   da.layer_vrow0 = 0;
-  da.chunk = 256;
-  da.max_splits = (max_ctx + 255) / 256;
+  int sms = 0, dev = 0;
+  CU(cudaGetDevice(&dev));
+  CU(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
+  da.chunk = decode_chunk(B, n_kv, max_ctx, sms);
+  da.max_splits = (max_ctx + da.chunk - 1) / da.chunk;
   da.part_o = reinterpret_cast<float*>(workspace);
   da.part_ml = da.part_o + (size_t)B * n_kv * da.max_splits * 16 * head_dim;
   da.out = reinterpret_cast<bf16*>(out);

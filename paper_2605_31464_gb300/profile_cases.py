@@ -3,6 +3,7 @@
     python -m paper_2605_31464_gb300.profile_cases gemm --M 8192 --N 37888 --K 3584 --mode swiglu
     python -m paper_2605_31464_gb300.profile_cases decode_attn --B 128 --ctx 3072 --n_q 28 --n_kv 4
     python -m paper_2605_31464_gb300.profile_cases prefill --workload 7b_prefill --batch 2 --layers 2
+    python -m paper_2605_31464_gb300.profile_cases forecast --workload 7b_prefill --layers 4 --n_decode 16
 
 Each case launches the kernel `--repeat` times on synthetic data through
 the C ABI and prints the mean CUDA-event time and the algorithmic rate.
@@ -73,7 +74,7 @@ def _prefill(a):
     import torch
     import synth
     import paper_2605_31464_gb300 as gf
-    w = synth.workload(a.workload, batch=a.batch)
+    w = synth.workload(a.workload, batch=a.batch or 2)
     shape = dataclasses.replace(w.model, layers=a.layers) if a.layers else w.model
     ids, off = synth.packed_prompts(w)
     dev = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
@@ -106,12 +107,57 @@ def _prefill(a):
     m.close()
 
 
+def _forecast(a):
+    """gf_forecast_batch on a workload with `--layers` layers (default all): prefill + decode + verdict."""
+    import dataclasses
+    import torch
+    import synth
+    import paper_2605_31464_gb300 as gf
+    w = synth.workload(a.workload, batch=a.batch or synth.workload(a.workload).batch)
+    shape = dataclasses.replace(w.model, layers=a.layers) if a.layers else w.model
+    n_dec = a.n_decode or w.n_decode
+    inc, io, cand, co = synth.prompts(w)
+    lens = np.diff(io) + np.diff(co)
+    dev = lambda bits: torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+    W = {"embed": dev(synth.embed_bf16(shape)), "lm_head": dev(synth.head_bf16(shape)),
+         "final_norm": dev(synth.ones_bf16(shape.d_model))}
+    for k in ("attn_norm", "wq", "wk", "wv", "wo", "ffn_norm", "w_gate", "w_up", "w_down"):
+        W[k] = []
+    for l in range(shape.layers):
+        for k, v in synth.layer_weights_bf16(shape, l).items():
+            W[k].append(dev(v))
+        W["attn_norm"].append(dev(synth.ones_bf16(shape.d_model)))
+        W["ffn_norm"].append(dev(synth.ones_bf16(shape.d_model)))
+    m = gf.Model(shape, W, max_batch=w.batch, max_seq=int(lens.max()) + n_dec,
+                 max_prefill_tokens=int(lens.sum()) + w.batch * n_dec + 64)
+    del W
+    inc_d, cand_d = torch.from_numpy(inc).cuda(), torch.from_numpy(cand).cuda()
+    s = torch.cuda.current_stream()
+    for r in range(a.repeat + 1):
+        if r == 1:
+            m.profile(1 << gf.GF_PROF_DECODE_STEPS)
+            m.profile_read(gf.GF_PROF_DECODE_STEPS)
+            e0 = torch.cuda.Event(enable_timing=True)
+            e0.record(s)
+        m.forecast_batch(inc_d, io, cand_d, co, n_dec, w.verdict_ids, w.tau, want_tokens=False)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e1.record(s)
+    torch.cuda.synchronize()
+    m.status()
+    ms = e0.elapsed_time(e1) / max(a.repeat, 1)
+    d = m.profile_read(gf.GF_PROF_DECODE_STEPS)
+    steps = max(a.repeat, 1) * max(n_dec - 1, 1)
+    print(f"forecast {a.workload} batch {w.batch} layers {shape.layers} n_decode {n_dec}: {ms:.2f} ms; "
+          f"decode step {d['ms'] / steps:.3f} ms, {d['bytes'] / (d['ms'] / 1e3) / 1e9 if d['ms'] else 0:.0f} GB/s")
+    m.close()
+
+
 def main(argv=None):
     root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
     if root not in sys.path:
         sys.path.insert(0, root)
     ap = argparse.ArgumentParser()
-    ap.add_argument("case", choices=["gemm", "decode_attn", "prefill"])
+    ap.add_argument("case", choices=["gemm", "decode_attn", "prefill", "forecast"])
     ap.add_argument("--M", type=int, default=8192)
     ap.add_argument("--N", type=int, default=37888)
     ap.add_argument("--K", type=int, default=3584)
@@ -125,13 +171,14 @@ def main(argv=None):
     ap.add_argument("--n_kv", type=int, default=4)
     ap.add_argument("--hd", type=int, default=128)
     ap.add_argument("--workload", default="7b_prefill")
-    ap.add_argument("--batch", type=int, default=2)
+    ap.add_argument("--batch", type=int, default=0)
     ap.add_argument("--layers", type=int, default=0)
     ap.add_argument("--repeat", type=int, default=3)
+    ap.add_argument("--n_decode", type=int, default=0)
     a = ap.parse_args(argv)
     from paper_2605_31464_gb300 import _build
     _build.build()
-    {"gemm": _gemm, "decode_attn": _decode_attn, "prefill": _prefill}[a.case](a)
+    {"gemm": _gemm, "decode_attn": _decode_attn, "prefill": _prefill, "forecast": _forecast}[a.case](a)
 
 
 if __name__ == "__main__":
