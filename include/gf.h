@@ -149,6 +149,23 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
                       const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
                       int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, float* final_logits, void* stream);
 
+/* gf_forecast_batch for a batch whose candidates all share one incumbent, as
+ * the candidates of one search step share the reference kernel r of
+ * x_i = (r, k_i, h) (Sec. 2.1): prompt_i = prefix ‖ candidate_i.  The
+ * prefix's full 64-token pages are prefilled once and every candidate's block
+ * table points at them (the pages are reference-counted); the remaining
+ * prefix_len % 64 tokens are prefilled with each candidate.  Results are those
+ * of gf_forecast_batch with inc_ids = the prefix for every item.
+ *   prefix_ids   device int32[prefix_len], prefix_len >= 0
+ *   cand_ids     device int32, packed; cand_offsets host int32[B+1]
+ *   every prompt needs at least one token after the shared pages;
+ *   other arguments as in gf_forecast_batch. */
+int gf_forecast_batch_shared(gf_model* m, int32_t B, const int32_t* prefix_ids, int32_t prefix_len,
+                             const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                             const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                             int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, float* final_logits,
+                             void* stream);
+
 /* gf_forecast_batch with every array in host memory: copies the ids to the
  * device, runs the forecast, copies p/conf/verdict_arg/defer (and tokens if
  * non-NULL) back, and synchronises `stream` before returning. */
@@ -270,6 +287,9 @@ int gf_debug_read_kv(gf_model* m, int32_t layer, int32_t handle, int32_t start, 
 /* Synchronise `stream` and report a device-side timeout recorded by any
  * kernel of this model since the last call (GF_ETIMEOUT), then clear it. */
 int gf_device_status(gf_model* m, void* stream);
+
+/* Pages of the KV pool not referenced by any live sequence. */
+int64_t gf_free_pages(const gf_model* m);
 
 /* Number of kernels this model has launched since creation (for accounting). */
 int64_t gf_launch_count(const gf_model* m);

@@ -46,7 +46,7 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
-           "gf_decode_attention_static"]
+           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN, GF_PROF_DECODE_STEPS = range(5)
@@ -72,6 +72,9 @@ def load(path: str = LIB_PATH):
                               ctypes.c_int),
         "gf_forecast_batch_host": ([_p, _c_i32, _p, _p, _p, _p, _c_i32, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p, _p],
                                    ctypes.c_int),
+        "gf_forecast_batch_shared": ([_p, _c_i32, _p, _c_i32, _p, _p, _c_i32, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p,
+                                      _p, _p], ctypes.c_int),
+        "gf_free_pages": ([_p], _c_i64),
         "gf_verdict": ([_c_i32, _p, _c_i64, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_debug_capture": ([_p, _c_i32, _c_i32, _p, _c_i64], ctypes.c_int),
         "gf_debug_read_kv": ([_p, _c_i32, _c_i32, _c_i32, _c_i32, _p, _p, _p], ctypes.c_int),
@@ -137,6 +140,17 @@ def gf_forecast_batch_host(model, B, inc_ids, inc_offsets, cand_ids, cand_offset
                            conf, verdict_arg, defer, tokens, stream):
     _check(load().gf_forecast_batch_host(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode,
                                          verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens, stream))
+
+
+def gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_offsets, n_decode, verdict_ids, K, tau,
+                             p, conf, verdict_arg, defer, tokens, final_logits, stream):
+    _check(load().gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_offsets, n_decode,
+                                           verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens, final_logits,
+                                           stream))
+
+
+def gf_free_pages(model) -> int:
+    return int(load().gf_free_pages(model))
 
 
 def gf_verdict(B, logits, ld, verdict_ids, K, tau, p, conf, verdict_arg, defer, stream):
@@ -325,6 +339,28 @@ class Model:
                           toks.data_ptr() if toks is not None and n_decode > 0 else None,
                           lg.data_ptr() if lg is not None else None, self.s)
         return dict(p=p, conf=conf, arg=arg, defer=defer, tokens=toks, logits=lg)
+
+    def forecast_batch_shared(self, prefix_ids, cand_ids, cand_offsets, n_decode, verdict_ids, tau, want_tokens=True,
+                              want_logits=False):
+        """Forecasts for candidates that all share one incumbent prefix (prefilled once)."""
+        torch = self.torch
+        co, vid = _i32_host(cand_offsets), _i32_host(verdict_ids)
+        B, K = len(co) - 1, len(vid)
+        p = torch.empty(B, K, dtype=torch.float32, device="cuda")
+        conf = torch.empty(B, dtype=torch.float32, device="cuda")
+        arg = torch.empty(B, dtype=torch.int32, device="cuda")
+        defer = torch.empty(B, dtype=torch.uint8, device="cuda")
+        toks = torch.empty(B, max(n_decode, 1), dtype=torch.int32, device="cuda") if want_tokens else None
+        lg = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
+        gf_forecast_batch_shared(self.handle, B, prefix_ids.data_ptr() if prefix_ids.numel() else None,
+                                 int(prefix_ids.numel()), cand_ids.data_ptr() if cand_ids.numel() else None, _ptr(co),
+                                 n_decode, _ptr(vid), K, float(tau), p.data_ptr(), conf.data_ptr(), arg.data_ptr(),
+                                 defer.data_ptr(), toks.data_ptr() if toks is not None and n_decode > 0 else None,
+                                 lg.data_ptr() if lg is not None else None, self.s)
+        return dict(p=p, conf=conf, arg=arg, defer=defer, tokens=toks, logits=lg)
+
+    def free_pages(self) -> int:
+        return gf_free_pages(self.handle)
 
     def forecast_batch_host(self, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, tau,
                             want_tokens=True):

@@ -76,10 +76,12 @@ __global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_co
   const int q0 = item.y * C::BQ;
   const int seq_start = a.offsets[b];
   const int len = a.offsets[b + 1] - seq_start;
+  const int past = a.past ? a.past[b] : 0;  // keys already cached before this prompt's first token
   const int kvh = head / (a.n_q / a.n_kv);
   const int32_t* pages = a.block_table + (int64_t)a.slots[b] * a.max_pages;
-  const int n_pages = (len + 63) >> 6;
-  const int n_tiles = (min(q0 + C::BQ, len) + C::BKV - 1) / C::BKV;
+  const int n_keys = past + len;
+  const int n_pages = (n_keys + 63) >> 6;
+  const int n_tiles = (past + min(q0 + C::BQ, len) + C::BKV - 1) / C::BKV;
 
   if (threadIdx.x == 0) {
     mbar_init(q_full, 1);
@@ -200,7 +202,7 @@ __global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_co
     // -------------------------------------------------------------- softmax warps 2..5
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;  // query row within the tile = TMEM lane
-    const int qpos = q0 + r;
+    const int qpos = past + q0 + r;  // absolute position of this query row
     const uint32_t lane_off = (uint32_t)(quarter * 32) << 16;
     const uint32_t o_addr = tmem + lane_off + C::O_COL;
     float m_ref = -INFINITY, l_run = 0.f;
@@ -222,8 +224,8 @@ __global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_co
       mbar_arrive(&s_free[st]);
       const int key0 = j * C::BKV;
       // causal / length mask only on the diagonal and last tiles (warp-uniform branch)
-      if ((key0 + C::BKV - 1 > q0) || (key0 + C::BKV > len)) {
-        const int lim = min(qpos + 1, len) - key0;  // keys [0, lim) of this tile are visible
+      if ((key0 + C::BKV - 1 > past + q0) || (key0 + C::BKV > n_keys)) {
+        const int lim = min(qpos + 1, n_keys) - key0;  // keys [0, lim) of this tile are visible
 #pragma unroll
         for (int i = 0; i < C::BKV; ++i)
           if (i >= lim) v[i] = __float_as_uint(-INFINITY);
@@ -291,13 +293,14 @@ __global__ void __launch_bounds__(192, 1) attn_prefill_tc_kernel(const __grid_co
     if (ok && wait_o(n_tiles - 1)) {
       tc_fence_after();
       const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-      uint4* dst = reinterpret_cast<uint4*>(a.out + (int64_t)(seq_start + (qpos < len ? qpos : 0)) * a.ldo + head * HD);
+      const int qrow = q0 + r;  // row of this query among the prompt's packed tokens
+      uint4* dst = reinterpret_cast<uint4*>(a.out + (int64_t)(seq_start + (qrow < len ? qrow : 0)) * a.ldo + head * HD);
 #pragma unroll 1
       for (int c = 0; c < HD / 32; ++c) {
         uint32_t ov[32];
         tmem_ld32(o_addr + c * 32, ov);
         tmem_ld_wait();
-        if (qpos < len) {
+        if (qrow < len) {
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             dst[c * 4 + q] = make_uint4(

@@ -104,7 +104,7 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
       if (a.offsets[mid] <= t) lo = mid; else hi = mid - 1;
     }
     slot = a.slots[lo];
-    pos = t - a.offsets[lo];
+    pos = t - a.offsets[lo] + (a.past ? a.past[lo] : 0);
   } else {
     slot = a.handles[t];
     pos = a.seq_len[slot];
@@ -281,16 +281,17 @@ cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t
 }
 
 // ------------------------------------------------------------------ bookkeeping
-__global__ void set_seq_len_kernel(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len) {
+__global__ void set_seq_len_kernel(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
+                                   const int32_t* past) {
   pdl_trigger();
   pdl_wait();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B) seq_len[slots[b]] = offsets[b + 1] - offsets[b];
+  if (b < B) seq_len[slots[b]] = offsets[b + 1] - offsets[b] + (past ? past[b] : 0);
 }
 cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
-                               cudaStream_t s) {
+                               cudaStream_t s, const int32_t* past) {
   if (B <= 0) return cudaSuccess;
-  return launch_pdl(set_seq_len_kernel, dim3((B + 255) / 256), dim3(256), 0, s, offsets, slots, B, seq_len);
+  return launch_pdl(set_seq_len_kernel, dim3((B + 255) / 256), dim3(256), 0, s, offsets, slots, B, seq_len, past);
 }
 
 // seq_len[handles[b]] += 1 for every b; *step += 1 when step is given (decode-step counter).
@@ -338,7 +339,7 @@ cudaError_t launch_finish_step(unsigned long long* keys, int B, int32_t* next, i
 // prompt_b = inc_ids[inc_off[b]:inc_off[b+1]] ++ cand_ids[cand_off[b]:cand_off[b+1]], packed at prompt_off[b].
 __global__ void build_prompts_kernel(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                      const int32_t* cand_off, const int32_t* prompt_off, int B, int T,
-                                     int32_t* out) {
+                                     int32_t* out, int shared_inc) {
   pdl_trigger();
   pdl_wait();
   for (int t = blockIdx.x * blockDim.x + threadIdx.x; t < T; t += gridDim.x * blockDim.x) {
@@ -348,18 +349,19 @@ __global__ void build_prompts_kernel(const int32_t* inc_ids, const int32_t* inc_
       if (prompt_off[mid] <= t) lo = mid; else hi = mid - 1;
     }
     const int j = t - prompt_off[lo];
-    const int n_inc = inc_off[lo + 1] - inc_off[lo];
-    out[t] = j < n_inc ? inc_ids[inc_off[lo] + j] : cand_ids[cand_off[lo] + (j - n_inc)];
+    const int n_inc = shared_inc >= 0 ? shared_inc : inc_off[lo + 1] - inc_off[lo];
+    const int inc0 = shared_inc >= 0 ? 0 : inc_off[lo];
+    out[t] = j < n_inc ? inc_ids[inc0 + j] : cand_ids[cand_off[lo] + (j - n_inc)];
   }
 }
 cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                  const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
-                                 cudaStream_t s) {
+                                 cudaStream_t s, int shared_inc) {
   if (T <= 0) return cudaSuccess;
   int blocks = (T + 255) / 256;
   if (blocks > 4096) blocks = 4096;
   return launch_pdl(build_prompts_kernel, dim3(blocks), dim3(256), 0, s, inc_ids, inc_off, cand_ids, cand_off,
-                    prompt_off, B, T, out);
+                    prompt_off, B, T, out, shared_inc);
 }
 
 // ------------------------------------------------------------------ weight packing

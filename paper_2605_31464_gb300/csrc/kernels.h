@@ -49,6 +49,7 @@ struct PrefillAttnArgs {
   const int2* items;          // (item, q_tile) work list, heaviest first
   const int32_t* offsets;     // [B+1] token offsets of the packed prompts
   const int32_t* slots;       // [B] sequence slot of each prompt
+  const int32_t* past;        // [B] positions already cached before this prompt's tokens, or nullptr
   const int32_t* block_table; // [slots][max_pages]
   int max_pages;
   int n_q, n_kv;
@@ -95,9 +96,11 @@ struct RopeKvArgs {
   bf16* k_cache;
   bf16* v_cache;
   const float2* rope_cs;      // [max_seq][hd/2] (cos, sin)
-  // prefill: offsets/slots describe the packed prompts; decode: offsets == nullptr
+  // prefill: offsets/slots (and past: cached positions before each prompt, or nullptr) describe the
+  // packed prompts; decode: offsets == nullptr
   const int32_t* offsets;
   const int32_t* slots;
+  const int32_t* past;
   int B;
   const int32_t* handles;
   const int32_t* seq_len;
@@ -120,7 +123,7 @@ cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t
 cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t* ids, int K, float tau, float* p,
                            float* conf, int32_t* arg, uint8_t* defer, cudaStream_t s);
 cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,
-                               cudaStream_t s);
+                               cudaStream_t s, const int32_t* past = nullptr);
 cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cudaStream_t s,
                            int32_t* step = nullptr);
 // Greedy tokens from the argmax keys of the LM-head GEMM: next[b] (and tok[b*stride + col],
@@ -129,9 +132,10 @@ cudaError_t launch_advance(const int32_t* handles, int B, int32_t* seq_len, cuda
 cudaError_t launch_finish_step(unsigned long long* keys, int B, int32_t* next, int32_t* tok, int64_t tok_stride,
                                int32_t* step, int col_base, int col_limit, const int32_t* handles,
                                int32_t* seq_len, cudaStream_t s);
+// shared_inc >= 0: every prompt starts with inc_ids[0 .. shared_inc) (inc_off unused).
 cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off, const int32_t* cand_ids,
                                  const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
-                                 cudaStream_t s);
+                                 cudaStream_t s, int shared_inc = -1);
 cudaError_t launch_pack_gate_up(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst, cudaStream_t s);
 cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStream_t s);
 cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cudaStream_t s);

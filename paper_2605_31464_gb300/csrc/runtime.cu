@@ -186,6 +186,7 @@ struct gf_model {
   std::vector<int32_t> h_bt, h_len;
   std::vector<char> live;
   std::vector<int32_t> free_pages, free_slots;
+  std::vector<int32_t> page_ref;  // block-table entries that point at each page (shared prefixes)
   std::vector<Capture> caps;
   std::map<std::tuple<const void*, uint64_t, uint64_t, uint32_t>, CUtensorMap> maps;
   Staging staging;
@@ -384,25 +385,33 @@ int alloc_pages(gf_model* m, int slot, int first, int count, std::vector<std::pa
     const int p = m->free_pages.back();
     m->free_pages.pop_back();
     m->h_bt[(int64_t)slot * m->max_pages + j] = p;
+    m->page_ref[p] = 1;
     undo->push_back({slot, j});
   }
   return GF_OK;
 }
 
-void undo_pages(gf_model* m, const std::vector<std::pair<int, int>>& undo) {
-  for (auto it = undo.rbegin(); it != undo.rend(); ++it) {
-    int32_t& e = m->h_bt[(int64_t)it->first * m->max_pages + it->second];
-    m->free_pages.push_back(e);
-    e = -1;
+// Point entries [0, count) of `slot` at the pages of `from` (copy-free sharing of a cached prefix).
+void share_pages(gf_model* m, int slot, int from, int count, std::vector<std::pair<int, int>>* undo) {
+  for (int j = 0; j < count; ++j) {
+    const int p = m->h_bt[(int64_t)from * m->max_pages + j];
+    m->h_bt[(int64_t)slot * m->max_pages + j] = p;
+    m->page_ref[p] += 1;
+    undo->push_back({slot, j});
   }
 }
 
+void drop_page(gf_model* m, int32_t& e) {
+  if (e >= 0 && --m->page_ref[e] == 0) m->free_pages.push_back(e);
+  e = -1;
+}
+
+void undo_pages(gf_model* m, const std::vector<std::pair<int, int>>& undo) {
+  for (auto it = undo.rbegin(); it != undo.rend(); ++it) drop_page(m, m->h_bt[(int64_t)it->first * m->max_pages + it->second]);
+}
+
 void release_slot(gf_model* m, int slot) {
-  for (int j = 0; j < m->max_pages; ++j) {
-    int32_t& e = m->h_bt[(int64_t)slot * m->max_pages + j];
-    if (e >= 0) m->free_pages.push_back(e);
-    e = -1;
-  }
+  for (int j = 0; j < m->max_pages; ++j) drop_page(m, m->h_bt[(int64_t)slot * m->max_pages + j]);
   m->h_len[slot] = 0;
   m->live[slot] = 0;
   m->free_slots.push_back(slot);
@@ -414,17 +423,21 @@ int upload_block_table(gf_model* m, cudaStream_t s) {
 
 // Prefill of B packed prompts already on the device.  `reserve` extra
 // tokens of KV pages are allocated per sequence (decode steps to come).
+// past > 0: every prompt continues a cached prefix of `past` positions (a multiple of 64) whose
+// pages belong to slot `share_slot`; the prompt's tokens sit at positions past, past+1, ...
+// want_head = false skips the final norm, LM head and greedy token (prefix-only prefill).
 int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets, int reserve, int32_t* handles_out,
                  float* logits_dst, int32_t* next_dst, cudaStream_t s, int32_t* tokens_col = nullptr,
-                 int64_t tokens_stride = 0) {
+                 int64_t tokens_stride = 0, int past = 0, int share_slot = -1, bool want_head = true) {
   if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
   if (!ids || !offsets) return fail(GF_EINVAL, "null ids or offsets");
   if (offsets[0] != 0) return fail(GF_EINVAL, "offsets[0] must be 0");
   for (int b = 0; b < B; ++b) {
     const int len = offsets[b + 1] - offsets[b];
     if (len < 1) return fail(GF_EINVAL, "prompt %d has length %d", b, len);
-    if (len + reserve > m->cfg.max_seq)
-      return fail(GF_ECAPACITY, "prompt %d: %d tokens (+%d) exceed max_seq %d", b, len, reserve, m->cfg.max_seq);
+    if (past + len + reserve > m->cfg.max_seq)
+      return fail(GF_ECAPACITY, "prompt %d: %d tokens (+%d) exceed max_seq %d", b, past + len, reserve,
+                  m->cfg.max_seq);
   }
   const int64_t T = offsets[B];
   if (T > m->T_max) return fail(GF_ECAPACITY, "%lld prompt tokens exceed max_prefill_tokens %lld", (long long)T,
@@ -437,9 +450,11 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     slots[b] = m->free_slots.back();
     m->free_slots.pop_back();
   }
+  const int shared = past / 64;
   for (int b = 0; b < B; ++b) {
     const int len = offsets[b + 1] - offsets[b];
-    const int rc = alloc_pages(m, slots[b], 0, (len + reserve + 63) / 64, &undo);
+    if (shared > 0) share_pages(m, slots[b], share_slot, shared, &undo);
+    const int rc = alloc_pages(m, slots[b], shared, (past + len + reserve + 63) / 64 - shared, &undo);
     if (rc != GF_OK) {
       undo_pages(m, undo);
       for (int bb = B - 1; bb >= 0; --bb) m->free_slots.push_back(slots[bb]);
@@ -448,13 +463,14 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   }
   for (int b = 0; b < B; ++b) {
     m->live[slots[b]] = 1;
-    m->h_len[slots[b]] = offsets[b + 1] - offsets[b];
+    m->h_len[slots[b]] = past + offsets[b + 1] - offsets[b];
     handles_out[b] = slots[b];
   }
-  // descriptor: offsets | slots | work items (heaviest first)
+  // descriptor: offsets | slots | past | work items (heaviest first)
   std::vector<int32_t> desc;
   desc.insert(desc.end(), offsets, offsets + B + 1);
   desc.insert(desc.end(), slots.begin(), slots.end());
+  desc.insert(desc.end(), (size_t)B, past);
   const size_t items_at = desc.size() + (desc.size() & 1);  // int2 alignment
   desc.resize(items_at);
   std::vector<std::pair<int, int>> items;
@@ -465,7 +481,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   std::stable_sort(items.begin(), items.end(), [&](const std::pair<int, int>& x, const std::pair<int, int>& y) {
     auto cost = [&](const std::pair<int, int>& it) {
       const int len = offsets[it.first + 1] - offsets[it.first];
-      return std::min(it.second * 128 + 128, len);
+      return past + std::min(it.second * 128 + 128, len);
     };
     return cost(x) > cost(y);
   });
@@ -478,6 +494,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   TRY(upload_block_table(m, s));
   const int32_t* d_off = m->call;
   const int32_t* d_slots = m->call + B + 1;
+  const int32_t* d_past = past > 0 ? m->call + 2 * B + 1 : nullptr;
   const int2* d_items = reinterpret_cast<const int2*>(m->call + items_at);
 
   CU(gf::launch_embed(ids, (int)T, m->embed, m->vocab, m->d, m->resid, m->err, s));
@@ -501,6 +518,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     ra.rope_cs = m->rope_cs;
     ra.offsets = d_off;
     ra.slots = d_slots;
+    ra.past = d_past;
     ra.B = B;
     ra.block_table = m->bt;
     ra.max_pages = m->max_pages;
@@ -516,6 +534,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     pa.items = d_items;
     pa.offsets = d_off;
     pa.slots = d_slots;
+    pa.past = d_past;
     pa.block_table = m->bt;
     pa.max_pages = m->max_pages;
     pa.n_q = m->nq;
@@ -530,7 +549,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
       double pairs = 0;
       for (int b = 0; b < B; ++b) {
         const double n = offsets[b + 1] - offsets[b];
-        pairs += n * (n + 1) / 2;
+        pairs += n * (n + 1) / 2 + n * past;
       }
       ProfScope ps(m, s, GF_PROF_PREFILL_ATTN, pairs * m->nq * 4.0 * m->hd,
                    (double)T * (m->q_dim * 2 + 2 * m->nkv * m->hd * 2 + m->q_dim * 2));
@@ -545,6 +564,11 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     TRY(gemm(m, m->act, (int)T, m->ffn_pad, W.down, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, m->ffn));
   }
   TRY(fire_captures(m, m->L, m->resid, offsets, B, false, s));
+  if (!want_head) {
+    CU(gf::launch_set_seq_len(d_off, d_slots, B, m->seq_len, s, d_past));
+    m->launches++;
+    return GF_OK;
+  }
   CU(gf::launch_last_rows(d_off, B, m->last_idx, s));
   CU(gf::launch_rmsnorm(m->resid, m->d, m->last_idx, B, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
   m->launches += 2;
@@ -560,7 +584,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
       CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s));
     m->launches++;
   }
-  CU(gf::launch_set_seq_len(d_off, d_slots, B, m->seq_len, s));
+  CU(gf::launch_set_seq_len(d_off, d_slots, B, m->seq_len, s, d_past));
   m->launches++;
   return GF_OK;
 }
@@ -732,6 +756,60 @@ int prepare_decode(gf_model* m, int B, const int32_t* h, cudaStream_t s) {
 
 }  // namespace
 
+// The part of a forecast after the prefill: n_decode greedy steps (the first eager, the rest one
+// replayed CUDA graph), the verdict on the final logits, and the release of the sequences.
+int decode_verdict_release(gf_model* m, int B, std::vector<int32_t>& h, int n_decode, const int32_t* verdict_ids,
+                           int K, float tau, float* p, float* conf, int32_t* verdict_arg, uint8_t* defer,
+                           int32_t* tokens, float* final_logits, float* lg, cudaStream_t s) {
+  int rc = upload(m->staging, m->handles, h.data(), (size_t)B * sizeof(int32_t), s);
+  if (rc == GF_OK && n_decode > 0) {
+    lg = m->logits;
+    if (cudaMemsetAsync(m->ctl, 0, sizeof(int32_t), s) != cudaSuccess) rc = fail(GF_ECUDA, "memset failed");
+    // the first step runs eagerly (it also configures the kernels); the rest replay one captured graph
+    if (rc == GF_OK) rc = decode_impl(m, B, h.data(), m->next, m->logits, m->next, m->tok_hist, m->tok_stride, s, m->ctl);
+    if (rc == GF_OK && n_decode > 1) {
+      cudaGraphExec_t exec = nullptr;
+      rc = decode_graph(m, B, h.data(), &exec);
+      // algorithmic bytes of the replayed steps: every weight once per step, the cached K/V each
+      // sequence reads, and the new K/V rows written
+      double bytes = 0;
+      if (m->prof_mask & (1u << GF_PROF_DECODE_STEPS)) {
+        const double kv_tok = (double)m->L * m->nkv * m->hd * 2 * 2;
+        for (int step = 1; step < n_decode; ++step) {
+          double ctx = 0;
+          for (int b = 0; b < B; ++b) ctx += m->h_len[h[b]] + step;  // context of this step's query
+          bytes += m->weight_bytes + ctx * kv_tok + (double)B * kv_tok;
+        }
+      }
+      {
+        ProfScope ps(m, s, GF_PROF_DECODE_STEPS, 0.0, bytes);
+        for (int step = 1; step < n_decode && rc == GF_OK; ++step) {
+          const cudaError_t e = cudaGraphLaunch(exec, s);
+          if (e != cudaSuccess) rc = fail(GF_ECUDA, "graph launch failed: %s", cudaGetErrorString(e));
+          m->launches += m->graph_launches_per_step;
+        }
+      }
+      if (rc == GF_OK)
+        for (int b = 0; b < B; ++b) m->h_len[h[b]] += n_decode - 1;
+    }
+    if (rc == GF_OK && final_logits &&
+        cudaMemcpyAsync(final_logits, m->logits, (size_t)B * m->vocab * sizeof(float), cudaMemcpyDeviceToDevice,
+                        s) != cudaSuccess)
+      rc = fail(GF_ECUDA, "logits copy failed");
+  }
+  if (rc == GF_OK && tokens && n_decode > 0 &&
+      cudaMemcpy2DAsync(tokens, (size_t)n_decode * sizeof(int32_t), m->tok_hist, (size_t)m->tok_stride * sizeof(int32_t),
+                        (size_t)n_decode * sizeof(int32_t), B, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
+    rc = fail(GF_ECUDA, "tokens copy failed");
+  if (rc == GF_OK) {
+    const cudaError_t e = gf::launch_verdict(lg, m->vocab, B, verdict_ids, K, tau, p, conf, verdict_arg, defer, s);
+    if (e != cudaSuccess) rc = fail(GF_ECUDA, "verdict launch: %s", cudaGetErrorString(e));
+    m->launches++;
+  }
+  for (int b = 0; b < B; ++b) release_slot(m, h[b]);
+  return rc;
+}
+
 // Helpers for entry points defined in other translation units.
 namespace gf {
 // Tensor map over a KV pool viewed as `rows` rows of hd bf16 (boxes of 64 x 64); 0 on success.
@@ -773,6 +851,8 @@ extern "C" {
 const char* gf_last_error(void) { return g_err.c_str(); }
 
 int64_t gf_launch_count(const gf_model* m) { return m ? m->launches : 0; }
+
+int64_t gf_free_pages(const gf_model* m) { return m ? (int64_t)m->free_pages.size() : 0; }
 
 void gf_destroy(gf_model* m) {
   if (!m) return;
@@ -876,7 +956,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->last_idx, Bm);
   if (!rc) rc = dalloc(m, &m->next, Bm);
   if (!rc) rc = dalloc(m, &m->handles, Bm);
-  m->call_ints = 2 * Bm + 8 + 2 * (size_t)(T / 128 + Bm + 8);
+  m->call_ints = 3 * Bm + 8 + 2 * (size_t)(T / 128 + Bm + 8);
   if (!rc) rc = dalloc(m, &m->call, m->call_ints);
   if (!rc) rc = dalloc(m, &m->fcall, 3 * Bm + 8);
   if (!rc) rc = dalloc(m, &m->out_small, Bm * 12);
@@ -930,6 +1010,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   m->h_len.assign(m->B_max, 0);
   m->live.assign(m->B_max, 0);
   m->free_pages.reserve(m->num_pages);
+  m->page_ref.assign(m->num_pages, 0);
   for (int64_t p = m->num_pages - 1; p >= 0; --p) m->free_pages.push_back((int32_t)p);
   for (int sl = m->B_max - 1; sl >= 0; --sl) m->free_slots.push_back(sl);
   const uint64_t rows = (uint64_t)m->L * m->num_pages * m->nkv * 64;
@@ -1015,53 +1096,60 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
   // tok_hist[b, s] is the input of decode step s: the arg max of the logits before it
   TRY(prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), lg, m->next, s, m->tok_hist,
                    m->tok_stride));
-  int rc = upload(m->staging, m->handles, h.data(), (size_t)B * sizeof(int32_t), s);
-  if (rc == GF_OK && n_decode > 0) {
-    lg = m->logits;
-    if (cudaMemsetAsync(m->ctl, 0, sizeof(int32_t), s) != cudaSuccess) rc = fail(GF_ECUDA, "memset failed");
-    // the first step runs eagerly (it also configures the kernels); the rest replay one captured graph
-    if (rc == GF_OK) rc = decode_impl(m, B, h.data(), m->next, m->logits, m->next, m->tok_hist, m->tok_stride, s, m->ctl);
-    if (rc == GF_OK && n_decode > 1) {
-      cudaGraphExec_t exec = nullptr;
-      rc = decode_graph(m, B, h.data(), &exec);
-      // algorithmic bytes of the replayed steps: every weight once per step, the cached K/V each
-      // sequence reads, and the new K/V rows written
-      double bytes = 0;
-      if (m->prof_mask & (1u << GF_PROF_DECODE_STEPS)) {
-        const double kv_tok = (double)m->L * m->nkv * m->hd * 2 * 2;
-        for (int step = 1; step < n_decode; ++step) {
-          double ctx = 0;
-          for (int b = 0; b < B; ++b) ctx += m->h_len[h[b]] + step;  // context of this step's query
-          bytes += m->weight_bytes + ctx * kv_tok + (double)B * kv_tok;
-        }
-      }
-      {
-        ProfScope ps(m, s, GF_PROF_DECODE_STEPS, 0.0, bytes);
-        for (int step = 1; step < n_decode && rc == GF_OK; ++step) {
-          const cudaError_t e = cudaGraphLaunch(exec, s);
-          if (e != cudaSuccess) rc = fail(GF_ECUDA, "graph launch failed: %s", cudaGetErrorString(e));
-          m->launches += m->graph_launches_per_step;
-        }
-      }
-      if (rc == GF_OK)
-        for (int b = 0; b < B; ++b) m->h_len[h[b]] += n_decode - 1;
-    }
-    if (rc == GF_OK && final_logits &&
-        cudaMemcpyAsync(final_logits, m->logits, (size_t)B * m->vocab * sizeof(float), cudaMemcpyDeviceToDevice,
-                        s) != cudaSuccess)
-      rc = fail(GF_ECUDA, "logits copy failed");
+  return decode_verdict_release(m, B, h, n_decode, verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens,
+                                final_logits, lg, s);
+}
+
+int gf_forecast_batch_shared(gf_model* m, int32_t B, const int32_t* prefix_ids, int32_t prefix_len,
+                             const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                             const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
+                             int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, float* final_logits,
+                             void* stream) {
+  if (!m || !cand_offsets || !verdict_ids || !p || !conf || !verdict_arg || !defer)
+    return fail(GF_EINVAL, "null argument");
+  if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
+  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
+  if (!(tau >= 0.f && tau <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
+  if (n_decode < 0 || prefix_len < 0) return fail(GF_EINVAL, "negative length");
+  if (prefix_len > 0 && !prefix_ids) return fail(GF_EINVAL, "null prefix ids");
+  for (int k = 0; k < K; ++k)
+    if (verdict_ids[k] < 0 || verdict_ids[k] >= m->vocab) return fail(GF_EINVAL, "verdict id %d >= vocab", verdict_ids[k]);
+  if (cand_offsets[0] != 0) return fail(GF_EINVAL, "offsets must start at 0");
+  // full 64-token pages of the prefix are computed once and shared; its tail is part of every prompt
+  const int past = prefix_len / 64 * 64, tail = prefix_len - past;
+  std::vector<int32_t> poff(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int nc = cand_offsets[b + 1] - cand_offsets[b];
+    if (nc < 0 || tail + nc < 1) return fail(GF_EINVAL, "item %d: no tokens after the shared pages", b);
+    if (nc > 0 && !cand_ids) return fail(GF_EINVAL, "null ids");
+    poff[b + 1] = poff[b] + tail + nc;
   }
-  if (rc == GF_OK && tokens && n_decode > 0 &&
-      cudaMemcpy2DAsync(tokens, (size_t)n_decode * sizeof(int32_t), m->tok_hist, (size_t)m->tok_stride * sizeof(int32_t),
-                        (size_t)n_decode * sizeof(int32_t), B, cudaMemcpyDeviceToDevice, s) != cudaSuccess)
-    rc = fail(GF_ECUDA, "tokens copy failed");
-  if (rc == GF_OK) {
-    const cudaError_t e = gf::launch_verdict(lg, m->vocab, B, verdict_ids, K, tau, p, conf, verdict_arg, defer, s);
-    if (e != cudaSuccess) rc = fail(GF_ECUDA, "verdict launch: %s", cudaGetErrorString(e));
-    m->launches++;
+  if (poff[B] > m->T_max || past > m->T_max) return fail(GF_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
+  if (past > 0 && m->free_slots.size() < (size_t)B + 1) return fail(GF_ECAPACITY, "no free sequence slots");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int32_t hp = -1;
+  if (past > 0) {
+    const int32_t poff1[2] = {0, past};
+    TRY(prefill_impl(m, 1, prefix_ids, poff1, 0, &hp, nullptr, nullptr, s, nullptr, 0, 0, -1, false));
   }
-  for (int b = 0; b < B; ++b) release_slot(m, h[b]);
-  return rc;
+  std::vector<int32_t> desc;
+  desc.insert(desc.end(), cand_offsets, cand_offsets + B + 1);
+  desc.insert(desc.end(), poff.begin(), poff.end());
+  int rc = upload(m->staging, m->fcall, desc.data(), desc.size() * sizeof(int32_t), s);
+  if (rc == GF_OK &&
+      gf::launch_build_prompts(prefix_ids + past, nullptr, cand_ids, m->fcall, m->fcall + B + 1, B, poff[B],
+                               m->prompt_ids, s, tail) != cudaSuccess)
+    rc = fail(GF_ECUDA, "prompt assembly launch failed");
+  m->launches++;
+  std::vector<int32_t> h(B);
+  float* lg = (n_decode == 0 && final_logits) ? final_logits : m->logits;
+  if (rc == GF_OK)
+    rc = prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), lg, m->next, s, m->tok_hist,
+                      m->tok_stride, past, hp, true);
+  if (hp >= 0) release_slot(m, hp);  // the shared pages stay referenced by the candidates
+  TRY(rc);
+  return decode_verdict_release(m, B, h, n_decode, verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens,
+                                final_logits, lg, s);
 }
 
 int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
