@@ -253,6 +253,13 @@ int gf_decode_attention_static(const void* q, const void* k_cache, const void* v
                                int32_t max_ctx, int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out,
                                void* stream);
 
+/* Failure detection self-test: launch a kernel whose bounded wait on a barrier
+ * that nothing completes runs out after `limit_ms` (1..2000).  The kernel
+ * records the timeout and returns; this call synchronises `stream` and
+ * returns GF_ETIMEOUT when the device reported it (GF_OK would mean the wait
+ * did not run out).  The CUDA context stays usable. */
+int gf_selftest_timeout(uint32_t limit_ms, void* stream);
+
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes whose launches can be bracketed by CUDA events (on the
  * launching stream) for live timing inside a run. */

@@ -394,6 +394,23 @@ cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStrea
   return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ failure detection
+// Waits on a barrier that nothing completes: the bounded wait gives up after
+// limit_ns, records GF_ETIMEOUT in *err and the kernel returns normally.
+__global__ void timeout_probe_kernel(uint64_t limit_ns, int* err) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait_for(&bar, 0, limit_ns, err);
+}
+cudaError_t launch_timeout_probe(uint64_t limit_ns, int* err, cudaStream_t s) {
+  timeout_probe_kernel<<<1, 32, 0, s>>>(limit_ns, err);
+  return cudaGetLastError();
+}
+
 // ------------------------------------------------------------------ inspection
 __global__ void read_kv_kernel(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,
                                int slot, int start, int n, int n_kv, int hd, int64_t layer_row0, bf16* k_dst,

@@ -143,6 +143,8 @@ cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32
                            int slot, int start, int n, int n_kv, int hd, int64_t layer_row0, bf16* k_dst,
                            bf16* v_dst, cudaStream_t s);
 
+cudaError_t launch_timeout_probe(uint64_t limit_ns, int* err, cudaStream_t s);
+
 // Defined in runtime.cu for entry points of other translation units.
 // K cache: rows of hd, boxes {64, 64}; V cache (transposed pages): rows of 64 keys, boxes {64, hd}.
 int encode_kv_map(CUtensorMap* m, const void* base, int hd, uint64_t rows);

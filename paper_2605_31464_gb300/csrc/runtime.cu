@@ -1305,6 +1305,17 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   return GF_OK;
 }
 
+int gf_selftest_timeout(uint32_t limit_ms, void* stream) {
+  if (limit_ms < 1 || limit_ms > 2000) return fail(GF_EINVAL, "limit_ms outside 1..2000");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (!g_gemm_err) {
+    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
+    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
+  }
+  CU(gf::launch_timeout_probe((uint64_t)limit_ms * 1000000ull, g_gemm_err, s));
+  return gf_gemm_status(stream);
+}
+
 int gf_profile_enable(gf_model* m, uint32_t mask) {
   if (!m) return fail(GF_EINVAL, "null model");
   m->prof_mask = mask;
