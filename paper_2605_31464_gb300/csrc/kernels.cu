@@ -8,71 +8,149 @@ namespace gf {
 
 // ------------------------------------------------------------------ embedding
 // out[t, :] = float(table[ids[t], :]); an id outside [0, vocab) records
-// GF_EINVAL in the error word and yields a zero row.
-__global__ void embed_kernel(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err) {
+// GF_EINVAL in the error word and yields a zero row.  One block per token;
+// every thread issues all of its 16-byte loads before using them.
+constexpr int kRowThreads = 256;
+constexpr int kRowVec = 8;  // 16-byte vectors per thread: rows up to 256 * 8 * 4 = 8192 fp32 / 16384 bf16
+
+__global__ void __launch_bounds__(kRowThreads) embed_kernel(const int32_t* ids, int T, const bf16* table, int vocab,
+                                                            int d, float* out, int* err) {
   pdl_trigger();
   pdl_wait();
-  const int t = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
-  if (t >= T) return;
+  const int t = blockIdx.x;
   const int id = ids[t];
   float* dst = out + (int64_t)t * d;
+  const int nv = d / 8;  // uint4 (8 bf16) per row
   if (id < 0 || id >= vocab) {
-    if (lane == 0) atomicCAS(err, 0, 1);
-    for (int i = lane * 4; i < d; i += 128) *reinterpret_cast<float4*>(dst + i) = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (threadIdx.x == 0) atomicCAS(err, 0, 1);
+    for (int i = threadIdx.x * 4; i < d; i += kRowThreads * 4)
+      *reinterpret_cast<float4*>(dst + i) = make_float4(0.f, 0.f, 0.f, 0.f);
     return;
   }
-  const bf16* src = table + (int64_t)id * d;
-  for (int i = lane * 8; i < d; i += 256) {
-    const uint4 v = *reinterpret_cast<const uint4*>(src + i);
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v);
-    float2 f0 = __bfloat1622float2(h[0]), f1 = __bfloat1622float2(h[1]);
-    float2 f2 = __bfloat1622float2(h[2]), f3 = __bfloat1622float2(h[3]);
-    *reinterpret_cast<float4*>(dst + i) = make_float4(f0.x, f0.y, f1.x, f1.y);
-    *reinterpret_cast<float4*>(dst + i + 4) = make_float4(f2.x, f2.y, f3.x, f3.y);
+  const uint4* src = reinterpret_cast<const uint4*>(table + (int64_t)id * d);
+  uint4 v[kRowVec];
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int i = threadIdx.x + k * kRowThreads;
+    if (i < nv) v[k] = src[i];
+  }
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int i = threadIdx.x + k * kRowThreads;
+    if (i < nv) {
+      const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&v[k]);
+      const float2 f0 = __bfloat1622float2(h[0]), f1 = __bfloat1622float2(h[1]);
+      const float2 f2 = __bfloat1622float2(h[2]), f3 = __bfloat1622float2(h[3]);
+      *reinterpret_cast<float4*>(dst + i * 8) = make_float4(f0.x, f0.y, f1.x, f1.y);
+      *reinterpret_cast<float4*>(dst + i * 8 + 4) = make_float4(f2.x, f2.y, f3.x, f3.y);
+    }
   }
 }
 
 cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err,
                          cudaStream_t s) {
   if (T <= 0) return cudaSuccess;
-  return launch_pdl(embed_kernel, dim3((T + 7) / 8), dim3(256), 0, s, ids, T, table, vocab, d, out, err);
+  if (d % 8 || d > kRowThreads * kRowVec * 8) return cudaErrorInvalidValue;  // d <= 16384
+  return launch_pdl(embed_kernel, dim3(T), dim3(kRowThreads), 0, s, ids, T, table, vocab, d, out, err);
 }
 
 // ------------------------------------------------------------------ RMSNorm
 // y[r, :] = bf16(x[src, :] * rsqrt(mean(x[src, :]^2) + eps) * gain), src = row_idx ? row_idx[r] : r.
-__global__ void rmsnorm_kernel(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d,
-                               const float* gain, float eps, bf16* y, int64_t ldy) {
+// One block per row: every thread loads its float4s at once, the block reduces the sum of squares.
+__global__ void __launch_bounds__(kRowThreads) rmsnorm_kernel(const float* x, int64_t ldx, const int32_t* row_idx,
+                                                              int rows, int d, const float* gain, float eps, bf16* y,
+                                                              int64_t ldy) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float red[kRowThreads / 32];
+  const int r = blockIdx.x;
+  const int src = row_idx ? row_idx[r] : r;
+  const float4* xr = reinterpret_cast<const float4*>(x + (int64_t)src * ldx);
+  const int nv = d / 4;
+  float4 v[kRowVec];
+  float ss = 0.f;
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int i = threadIdx.x + k * kRowThreads;
+    v[k] = i < nv ? xr[i] : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  float tot = 0.f;
+#pragma unroll
+  for (int w = 0; w < kRowThreads / 32; ++w) tot += red[w];
+  const float inv = rsqrtf(tot / (float)d + eps);
+  uint2* yr = reinterpret_cast<uint2*>(y + (int64_t)r * ldy);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+#pragma unroll
+  for (int k = 0; k < kRowVec; ++k) {
+    const int i = threadIdx.x + k * kRowThreads;
+    if (i < nv) {
+      const float4 g = g4[i];
+      uint2 o;
+      o.x = pack_bf16(v[k].x * inv * g.x, v[k].y * inv * g.y);
+      o.y = pack_bf16(v[k].z * inv * g.z, v[k].w * inv * g.w);
+      yr[i] = o;
+    }
+  }
+}
+
+// Many rows (prefill): one warp per row, each lane's loads issued eight at a time.
+__global__ void __launch_bounds__(256) rmsnorm_warp_kernel(const float* x, int64_t ldx, const int32_t* row_idx,
+                                                           int rows, int d, const float* gain, float eps, bf16* y,
+                                                           int64_t ldy) {
   pdl_trigger();
   pdl_wait();
   const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (r >= rows) return;
   const int src = row_idx ? row_idx[r] : r;
-  const float* xr = x + (int64_t)src * ldx;
+  const float4* xr = reinterpret_cast<const float4*>(x + (int64_t)src * ldx);
+  const int nv = d / 4;
   float ss = 0.f;
-  for (int i = lane * 4; i < d; i += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + i);
-    ss += v.x * v.x + v.y * v.y + v.z * v.z + v.w * v.w;
+  for (int base = lane; base < nv; base += 8 * 32) {
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = base + k * 32 < nv ? xr[base + k * 32] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
   const float inv = rsqrtf(ss / (float)d + eps);
-  bf16* yr = y + (int64_t)r * ldy;
-  for (int i = lane * 4; i < d; i += 128) {
-    const float4 v = *reinterpret_cast<const float4*>(xr + i);
-    const float4 g = *reinterpret_cast<const float4*>(gain + i);
-    uint2 o;
-    o.x = pack_bf16(v.x * inv * g.x, v.y * inv * g.y);
-    o.y = pack_bf16(v.z * inv * g.z, v.w * inv * g.w);
-    *reinterpret_cast<uint2*>(yr + i) = o;
+  uint2* yr = reinterpret_cast<uint2*>(y + (int64_t)r * ldy);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+  for (int base = lane; base < nv; base += 8 * 32) {
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = base + k * 32 < nv ? xr[base + k * 32] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int i = base + k * 32;
+      if (i < nv) {
+        const float4 g = g4[i];
+        uint2 o;
+        o.x = pack_bf16(v[k].x * inv * g.x, v[k].y * inv * g.y);
+        o.y = pack_bf16(v[k].z * inv * g.z, v[k].w * inv * g.w);
+        yr[i] = o;
+      }
+    }
   }
 }
 
 cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
                            float eps, bf16* y, int64_t ldy, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
-  return launch_pdl(rmsnorm_kernel, dim3((rows + 7) / 8), dim3(256), 0, s, x, ldx, row_idx, rows, d, gain, eps, y, ldy);
+  if (d % 4) return cudaErrorInvalidValue;
+  if (rows >= 2048 || d > kRowThreads * kRowVec * 4)
+    return launch_pdl(rmsnorm_warp_kernel, dim3((rows + 7) / 8), dim3(256), 0, s, x, ldx, row_idx, rows, d, gain, eps,
+                      y, ldy);
+  return launch_pdl(rmsnorm_kernel, dim3(rows), dim3(kRowThreads), 0, s, x, ldx, row_idx, rows, d, gain, eps, y,
+                    ldy);
 }
 
 __global__ void last_rows_kernel(const int32_t* offsets, int B, int32_t* row_idx) {
@@ -115,34 +193,51 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
   const int in_page = pos & 63;
   float* src = a.qkv + (int64_t)t * a.ldqkv;
   const float2* cs = a.rope_cs + (int64_t)pos * half;
-  for (int idx = threadIdx.x; idx < heads * half; idx += blockDim.x) {
-    const int h = idx / half, i = idx % half;
-    const int c0 = h * a.hd + i;
-    const float x0 = src[c0], x1 = src[c0 + half];
-    if (a.zero_after) {
-      src[c0] = 0.f;
-      src[c0 + half] = 0.f;
-    }
-    if (h < a.n_q + a.n_kv) {
-      const float2 r = cs[i];
-      const bf16 y0 = __float2bfloat16(x0 * r.x - x1 * r.y);
-      const bf16 y1 = __float2bfloat16(x1 * r.x + x0 * r.y);
-      if (h < a.n_q) {
-        bf16* dst = a.q_out + (int64_t)t * a.ldq + h * a.hd;
-        dst[i] = y0;
-        dst[i + half] = y1;
-      } else {
-        const int g = h - a.n_q;
-        bf16* dst = a.k_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + g) * 64 + in_page) * a.hd;
-        dst[i] = y0;
-        dst[i + half] = y1;
+  const int n = heads * half;
+  // all of this thread's element pairs are loaded before any is used
+  constexpr int kU = 4;
+  for (int base = threadIdx.x; base < n; base += kU * blockDim.x) {
+    float x0[kU], x1[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx < n) {
+        const int c0 = (idx / half) * a.hd + idx % half;
+        x0[u] = src[c0];
+        x1[u] = src[c0 + half];
       }
-    } else {
-      // values are stored transposed per page: [page][kv head][hd][64 keys]
-      const int g = h - a.n_q - a.n_kv;
-      bf16* dst = a.v_cache + a.layer_row0 * a.hd + (((int64_t)page * a.n_kv + g) * a.hd + i) * 64 + in_page;
-      dst[0] = __float2bfloat16(x0);
-      dst[(int64_t)half * 64] = __float2bfloat16(x1);
+    }
+#pragma unroll
+    for (int u = 0; u < kU; ++u) {
+      const int idx = base + u * blockDim.x;
+      if (idx >= n) continue;
+      const int h = idx / half, i = idx % half;
+      const int c0 = h * a.hd + i;
+      if (a.zero_after) {
+        src[c0] = 0.f;
+        src[c0 + half] = 0.f;
+      }
+      if (h < a.n_q + a.n_kv) {
+        const float2 r = cs[i];
+        const bf16 y0 = __float2bfloat16(x0[u] * r.x - x1[u] * r.y);
+        const bf16 y1 = __float2bfloat16(x1[u] * r.x + x0[u] * r.y);
+        if (h < a.n_q) {
+          bf16* dst = a.q_out + (int64_t)t * a.ldq + h * a.hd;
+          dst[i] = y0;
+          dst[i + half] = y1;
+        } else {
+          const int g = h - a.n_q;
+          bf16* dst = a.k_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + g) * 64 + in_page) * a.hd;
+          dst[i] = y0;
+          dst[i + half] = y1;
+        }
+      } else {
+        // values are stored transposed per page: [page][kv head][hd][64 keys]
+        const int g = h - a.n_q - a.n_kv;
+        bf16* dst = a.v_cache + a.layer_row0 * a.hd + (((int64_t)page * a.n_kv + g) * a.hd + i) * 64 + in_page;
+        dst[0] = __float2bfloat16(x0[u]);
+        dst[(int64_t)half * 64] = __float2bfloat16(x1[u]);
+      }
     }
   }
 }
