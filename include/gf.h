@@ -180,6 +180,23 @@ int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const
 int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdict_ids, int32_t K, float tau,
                float* p, float* conf, int32_t* verdict_arg, uint8_t* defer, void* stream);
 
+/* What a search does with an 8-bin forecast (K = 8 verdict ids, one per speedup
+ * bin of Table tab:speedup-bins: S <= 0.25, (0.25,0.5], (0.5,0.71], (0.71,1],
+ * (1,1.41], (1.41,2], (2,4], > 4):
+ *   s_hat[i] = sum_b p[i,b] m_bins[b], the expected speedup that ranks
+ *              candidates (Sec. 3.1); m_bins host float[8] are the bin
+ *              representatives (m_2..m_7 = 0.35 0.59 0.84 1.19 1.68 2.83 in the
+ *              paper; m_1, m_8 are empirical means it does not print);
+ *   order[0..B) = candidate indices by decreasing s_hat, lower index first on
+ *              ties (measure the first ceil(c% * B) under a budget c);
+ *   disc[i]  = Pr[g >= x_cut], the discovery-moment score (Sec. 3.6): the mass
+ *              of the bins whose lower edge is >= x_cut;
+ *   disc_pred[i] = disc[i] >= tau_disc.
+ * p, s_hat, disc device float; order device int32; disc_pred device uint8.
+ * 1 <= B <= 1024.  Enqueued on `stream`. */
+int gf_select(int32_t B, const float* p, const float* m_bins, float x_cut, float tau_disc, float* s_hat,
+              int32_t* order, float* disc, uint8_t* disc_pred, void* stream);
+
 /* ---- building blocks --------------------------------------------------------
  * The dense contraction every projection of the forward pass uses, exposed on
  * its own: out[M,N] (op)= A[M,K] . W[N,K]^T on the tcgen05 tensor cores.

@@ -46,7 +46,7 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
-           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout"]
+           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN, GF_PROF_DECODE_STEPS = range(5)
@@ -76,6 +76,7 @@ def load(path: str = LIB_PATH):
                                       _p, _p], ctypes.c_int),
         "gf_free_pages": ([_p], _c_i64),
         "gf_selftest_timeout": ([ctypes.c_uint32, _p], ctypes.c_int),
+        "gf_select": ([_c_i32, _p, _p, _c_f32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_verdict": ([_c_i32, _p, _c_i64, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_debug_capture": ([_p, _c_i32, _c_i32, _p, _c_i64], ctypes.c_int),
         "gf_debug_read_kv": ([_p, _c_i32, _c_i32, _c_i32, _c_i32, _p, _p, _p], ctypes.c_int),
@@ -148,6 +149,25 @@ def gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_of
     _check(load().gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_offsets, n_decode,
                                            verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens, final_logits,
                                            stream))
+
+
+def gf_select(B, p, m_bins, x_cut, tau_disc, s_hat, order, disc, disc_pred, stream):
+    _check(load().gf_select(B, p, m_bins, x_cut, tau_disc, s_hat, order, disc, disc_pred, stream))
+
+
+def select(p, m_bins, x_cut, tau_disc, stream=None):
+    """Expected speedup, ranking and discovery score of a [B, 8] CUDA tensor of bin probabilities."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    B = p.shape[0]
+    m = np.ascontiguousarray(np.asarray(m_bins, dtype=np.float32))
+    s_hat = torch.empty(B, dtype=torch.float32, device=p.device)
+    order = torch.empty(B, dtype=torch.int32, device=p.device)
+    disc = torch.empty(B, dtype=torch.float32, device=p.device)
+    pred = torch.empty(B, dtype=torch.uint8, device=p.device)
+    gf_select(B, p.data_ptr(), m.ctypes.data_as(_p), float(x_cut), float(tau_disc), s_hat.data_ptr(),
+              order.data_ptr(), disc.data_ptr(), pred.data_ptr(), s.cuda_stream)
+    return s_hat, order, disc, pred
 
 
 def gf_selftest_timeout(limit_ms, stream):

@@ -489,6 +489,69 @@ cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStrea
   return cudaGetLastError();
 }
 
+// ------------------------------------------------------------------ selection (Sec. 3.1, 3.6)
+// One block of 1024 threads, B <= 1024 candidates with 8 bin probabilities each:
+//   s_hat[i] = sum_b p[i,b] m[b]; order = indices by decreasing s_hat (lower index first on ties,
+//   bitonic sort in shared memory); disc[i] = mass of the bins whose lower edge is >= x;
+//   disc_pred[i] = disc[i] >= tau.
+struct BinReps {
+  float m[8];
+};
+__global__ void __launch_bounds__(1024) select_kernel(int B, const float* p, BinReps reps, float x, float tau,
+                                                       float* s_hat, int32_t* order, float* disc,
+                                                       uint8_t* disc_pred) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ float key[1024];
+  __shared__ int idx[1024];
+  const float lower[8] = {0.f, 0.25f, 0.5f, 0.71f, 1.0f, 1.41f, 2.0f, 4.0f};
+  const int i = threadIdx.x;
+  float sv = -INFINITY;
+  if (i < B) {
+    float acc = 0.f, d = 0.f;
+#pragma unroll
+    for (int b = 0; b < 8; ++b) {
+      const float pb = p[(int64_t)i * 8 + b];
+      acc += pb * reps.m[b];
+      if (lower[b] >= x) d += pb;
+    }
+    sv = acc;
+    s_hat[i] = acc;
+    disc[i] = d;
+    disc_pred[i] = d >= tau ? 1 : 0;
+  }
+  key[i] = sv;
+  idx[i] = i < B ? i : 0x7fffffff;
+  __syncthreads();
+  // bitonic sort, "first" = larger key, then smaller index
+  for (int size = 2; size <= 1024; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const int j = i ^ stride;
+      if (j > i) {
+        const bool up = (i & size) == 0;
+        const float ka = key[i], kb = key[j];
+        const int ia = idx[i], ib = idx[j];
+        const bool a_first = ka > kb || (ka == kb && ia < ib);
+        if (a_first != up) {
+          key[i] = kb;
+          key[j] = ka;
+          idx[i] = ib;
+          idx[j] = ia;
+        }
+      }
+      __syncthreads();
+    }
+  }
+  if (i < B) order[i] = idx[i];
+}
+cudaError_t launch_select(int B, const float* p, const float* m_bins, float x, float tau, float* s_hat,
+                          int32_t* order, float* disc, uint8_t* disc_pred, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  BinReps r;
+  for (int b = 0; b < 8; ++b) r.m[b] = m_bins[b];
+  return launch_pdl(select_kernel, dim3(1), dim3(1024), 0, s, B, p, r, x, tau, s_hat, order, disc, disc_pred);
+}
+
 // ------------------------------------------------------------------ failure detection
 // Waits on a barrier that nothing completes: the bounded wait gives up after
 // limit_ns, records GF_ETIMEOUT in *err and the kernel returns normally.

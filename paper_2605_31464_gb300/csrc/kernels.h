@@ -144,6 +144,8 @@ cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32
                            bf16* v_dst, cudaStream_t s);
 
 cudaError_t launch_timeout_probe(uint64_t limit_ns, int* err, cudaStream_t s);
+cudaError_t launch_select(int B, const float* p, const float* m_bins, float x, float tau, float* s_hat,
+                          int32_t* order, float* disc, uint8_t* disc_pred, cudaStream_t s);
 
 // Defined in runtime.cu for entry points of other translation units.
 // K cache: rows of hd, boxes {64, 64}; V cache (transposed pages): rows of 64 keys, boxes {64, hd}.

@@ -1305,6 +1305,16 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   return GF_OK;
 }
 
+int gf_select(int32_t B, const float* p, const float* m_bins, float x_cut, float tau_disc, float* s_hat,
+              int32_t* order, float* disc, uint8_t* disc_pred, void* stream) {
+  if (!p || !m_bins || !s_hat || !order || !disc || !disc_pred) return fail(GF_EINVAL, "null argument");
+  if (B < 1 || B > 1024) return fail(GF_EINVAL, "batch %d outside 1..1024", B);
+  if (!(tau_disc >= 0.f && tau_disc <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
+  CU(gf::launch_select(B, p, m_bins, x_cut, tau_disc, s_hat, order, disc, disc_pred,
+                       reinterpret_cast<cudaStream_t>(stream)));
+  return GF_OK;
+}
+
 int gf_selftest_timeout(uint32_t limit_ms, void* stream) {
   if (limit_ms < 1 || limit_ms > 2000) return fail(GF_EINVAL, "limit_ms outside 1..2000");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
