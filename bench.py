@@ -234,9 +234,12 @@ def run_ours(args):
     max_len = int(lens.max())
 
     W = device_weights(m)
-    # one slot more than the batch: the shared-incumbent path keeps the prefix in its own slot
-    model = gf.Model(m, W, max_batch=B + 1, max_seq=max_len + w.n_decode, max_prefill_tokens=int(lens.sum()) +
-                     B * w.n_decode + 64)
+    # one slot more than the batch: the shared-incumbent path keeps the prefix in its own slot;
+    # the sampled forecasts (3 repeats per item, Sec. 3.1 setup) need a slot per row
+    n_rep = 3
+    sample_rows = B * n_rep if (world == 1 and B * n_rep <= 128) else 0
+    model = gf.Model(m, W, max_batch=max(B + 1, sample_rows), max_seq=max_len + w.n_decode,
+                     max_prefill_tokens=int(lens.sum()) + B * w.n_decode + 64)
     del W
     torch.cuda.empty_cache()
     inc_d = torch.from_numpy(inc).cuda()
@@ -303,6 +306,29 @@ def run_ours(args):
                         "ms_per_step": ms_sh / args.steps,
                         "path": "gf_forecast_batch_shared: the incumbent's full 64-token pages are prefilled once per "
                                 "batch and shared through the block tables"}
+
+    # ---- temperature-1 sampling, three repeats per item (each prompt prefilled once, repeats fork its pages)
+    sampled = None
+    if sample_rows:
+        def step_sampled(seed):
+            return model.forecast_batch_sampled(inc_d, io, cand_d, co, w.n_decode, w.verdict_ids, w.tau,
+                                                repeats=n_rep, temperature=1.0, seed=seed, want_tokens=False)
+
+        step_sampled(0)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for k in range(args.steps):
+            step_sampled(k + 1)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        model.status()
+        ms_s = e0.elapsed_time(e1)
+        sampled = {"value": B * n_rep * args.steps / (ms_s / 1e3), "unit": "sampled forecasts/s",
+                   "items_per_s": B * args.steps / (ms_s / 1e3), "repeats": n_rep, "temperature": 1.0,
+                   "ms_per_step": ms_s / args.steps,
+                   "path": "gf_forecast_batch_sampled: each prompt is prefilled once and its repeats fork its KV "
+                           "pages; tokens are drawn by the Gumbel-max rule fused into the LM-head GEMM"}
 
     # ---- end to end through the host-buffer entry point (copies inside the timed region)
     model.forecast_batch_host(inc, io, cand, co, w.n_decode, w.verdict_ids, w.tau, want_tokens=True)
@@ -374,7 +400,7 @@ def run_ours(args):
             "roofline_secondary": secondary,
             "e2e": {"value": B * world * args.steps / e2e_s, "unit": "forecasts/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
-            "gpu_launches": int(launches), "clocks": clk, "prefix_reuse": prefix_reuse,
+            "gpu_launches": int(launches), "clocks": clk, "prefix_reuse": prefix_reuse, "sampled": sampled,
             "prefill_tok_per_s": float(lens.sum()) / (prefill_ms / 1e3),
             "decode_tok_per_s": B / (decode_ms / 1e3),
             "prefill_ms": prefill_ms, "decode_ms_per_step": decode_ms,

@@ -174,6 +174,37 @@ int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const
                            const int32_t* verdict_ids, int32_t K, float tau, float* p, float* conf,
                            int32_t* verdict_arg, uint8_t* defer, int32_t* tokens, void* stream);
 
+/* gf_forecast_batch with temperature sampling instead of greedy decoding, each
+ * item sampled `repeats` times (Sec. 3.1 setup: three repeats per row at
+ * temperature 1.0, reported as mean and population standard deviation).
+ *   Row r = i * repeats + j is repeat j of item i.  Each item's prompt is
+ *   prefilled once; its repeats share the prompt's full KV pages.
+ *   Token t of row r (t = 0 from the prompt's logits, t = s + 1 from decode
+ *   step s) is argmax_v (logits_v / temperature + G), G = -ln(-ln U) with U
+ *   from Philox4x64-10 under key (seed, 0) at counter (v, t, r / 4, 0), word
+ *   r mod 4, U = (floor(w / 2^41) + 1/2) 2^-23: an exact draw from
+ *   softmax(logits / temperature), reproducible from (seed, t, r, v) alone.
+ *   The verdict reads each row's final logits as in gf_forecast_batch.
+ *   repeats >= 1, B * repeats <= max_batch; temperature > 0 and finite.
+ *   p [B*repeats*K], conf, verdict_arg, defer [B*repeats]: per row, device.
+ *   p_mean, p_std [B*K], conf_mean, conf_std [B]: device float or NULL, the
+ *     mean and population standard deviation (divided by repeats) over the
+ *     repeats of each item.
+ *   tokens device int32[B*repeats*n_decode] or NULL; final_logits device
+ *     float[B*repeats*vocab] or NULL; other arguments as in gf_forecast_batch. */
+int gf_forecast_batch_sampled(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                              const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                              int32_t repeats, float temperature, uint64_t seed, const int32_t* verdict_ids,
+                              int32_t K, float tau, float* p, float* conf, int32_t* verdict_arg, uint8_t* defer,
+                              float* p_mean, float* p_std, float* conf_mean, float* conf_std, int32_t* tokens,
+                              float* final_logits, void* stream);
+
+/* Stand-alone temperature draw (the rule of gf_forecast_batch_sampled) on caller logits:
+ *   logits device float[B*ld], row b is sampled row r = b, token index t = token_index >= 0;
+ *   out_ids device int32[B].  V <= ld; temperature > 0 and finite. */
+int gf_sample_tokens(int32_t B, const float* logits, int64_t ld, int32_t V, uint64_t seed, int32_t token_index,
+                     float temperature, int32_t* out_ids, void* stream);
+
 /* Stand-alone verdict step (Sec. 2.1) on caller logits:
  *   logits device float[B*ld] (row stride ld >= max verdict id + 1);
  *   verdict_ids host int32[K]; outputs as in gf_forecast_batch. */

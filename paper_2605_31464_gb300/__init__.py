@@ -46,7 +46,8 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
-           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select"]
+           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select",
+           "gf_forecast_batch_sampled", "gf_sample_tokens"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN, GF_PROF_DECODE_STEPS = range(5)
@@ -74,6 +75,9 @@ def load(path: str = LIB_PATH):
                                    ctypes.c_int),
         "gf_forecast_batch_shared": ([_p, _c_i32, _p, _c_i32, _p, _p, _c_i32, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p,
                                       _p, _p], ctypes.c_int),
+        "gf_forecast_batch_sampled": ([_p, _c_i32, _p, _p, _p, _p, _c_i32, _c_i32, _c_f32, ctypes.c_uint64, _p, _c_i32,
+                                       _c_f32, _p, _p, _p, _p, _p, _p, _p, _p, _p, _p, _p], ctypes.c_int),
+        "gf_sample_tokens": ([_c_i32, _p, _c_i64, _c_i32, ctypes.c_uint64, _c_i32, _c_f32, _p, _p], ctypes.c_int),
         "gf_free_pages": ([_p], _c_i64),
         "gf_selftest_timeout": ([ctypes.c_uint32, _p], ctypes.c_int),
         "gf_select": ([_c_i32, _p, _p, _c_f32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
@@ -149,6 +153,28 @@ def gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_of
     _check(load().gf_forecast_batch_shared(model, B, prefix_ids, prefix_len, cand_ids, cand_offsets, n_decode,
                                            verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens, final_logits,
                                            stream))
+
+
+def gf_forecast_batch_sampled(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, repeats, temperature,
+                              seed, verdict_ids, K, tau, p, conf, verdict_arg, defer, p_mean, p_std, conf_mean,
+                              conf_std, tokens, final_logits, stream):
+    _check(load().gf_forecast_batch_sampled(model, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, repeats,
+                                            temperature, seed, verdict_ids, K, tau, p, conf, verdict_arg, defer,
+                                            p_mean, p_std, conf_mean, conf_std, tokens, final_logits, stream))
+
+
+def gf_sample_tokens(B, logits, ld, V, seed, token_index, temperature, out_ids, stream):
+    _check(load().gf_sample_tokens(B, logits, ld, V, seed, token_index, temperature, out_ids, stream))
+
+
+def sample_tokens(logits, seed, token_index, temperature, stream=None):
+    """Temperature draw (Gumbel-max, counter-based) for each row of a [B, V] float32 CUDA tensor."""
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    out = torch.empty(logits.shape[0], dtype=torch.int32, device=logits.device)
+    gf_sample_tokens(logits.shape[0], logits.data_ptr(), logits.stride(0), logits.shape[1], int(seed),
+                     int(token_index), float(temperature), out.data_ptr(), s.cuda_stream)
+    return out
 
 
 def gf_select(B, p, m_bins, x_cut, tau_disc, s_hat, order, disc, disc_pred, stream):
@@ -384,6 +410,31 @@ class Model:
                                  defer.data_ptr(), toks.data_ptr() if toks is not None and n_decode > 0 else None,
                                  lg.data_ptr() if lg is not None else None, self.s)
         return dict(p=p, conf=conf, arg=arg, defer=defer, tokens=toks, logits=lg)
+
+    def forecast_batch_sampled(self, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, tau,
+                               repeats=3, temperature=1.0, seed=0, want_tokens=True, want_logits=False):
+        """Forecasts by temperature sampling, `repeats` rows per item (row = item * repeats + repeat),
+        with the mean and population standard deviation of p and conf over each item's repeats."""
+        torch = self.torch
+        io, co, vid = _i32_host(inc_offsets), _i32_host(cand_offsets), _i32_host(verdict_ids)
+        B, K = len(io) - 1, len(vid)
+        BR = B * repeats
+        f32 = dict(dtype=torch.float32, device="cuda")
+        p, conf = torch.empty(BR, K, **f32), torch.empty(BR, **f32)
+        arg = torch.empty(BR, dtype=torch.int32, device="cuda")
+        defer = torch.empty(BR, dtype=torch.uint8, device="cuda")
+        p_mean, p_std = torch.empty(B, K, **f32), torch.empty(B, K, **f32)
+        conf_mean, conf_std = torch.empty(B, **f32), torch.empty(B, **f32)
+        toks = torch.empty(BR, max(n_decode, 1), dtype=torch.int32, device="cuda") if want_tokens else None
+        lg = torch.empty(BR, self.shape.vocab, **f32) if want_logits else None
+        gf_forecast_batch_sampled(self.handle, B, inc_ids.data_ptr(), _ptr(io), cand_ids.data_ptr(), _ptr(co),
+                                  n_decode, repeats, float(temperature), int(seed), _ptr(vid), K, float(tau),
+                                  p.data_ptr(), conf.data_ptr(), arg.data_ptr(), defer.data_ptr(), p_mean.data_ptr(),
+                                  p_std.data_ptr(), conf_mean.data_ptr(), conf_std.data_ptr(),
+                                  toks.data_ptr() if toks is not None and n_decode > 0 else None,
+                                  lg.data_ptr() if lg is not None else None, self.s)
+        return dict(p=p, conf=conf, arg=arg, defer=defer, p_mean=p_mean, p_std=p_std, conf_mean=conf_mean,
+                    conf_std=conf_std, tokens=toks, logits=lg)
 
     def free_pages(self) -> int:
         return gf_free_pages(self.handle)

@@ -53,7 +53,8 @@ static cudaError_t dispatch_swap(const CUtensorMap& tmA, const CUtensorMap& tmB,
 
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
-                        bool swap, unsigned long long* argmax_keys) {
+                        bool swap, unsigned long long* argmax_keys, const SampleParams* sample,
+                        const int32_t* sample_step, int sample_step_bias) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0) return cudaErrorInvalidValue;
   if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
@@ -81,6 +82,9 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   p.ldo = ldo;
   p.err = err;
   p.argmax_keys = (swap && mode == kStoreF32) ? argmax_keys : nullptr;
+  p.sample = p.argmax_keys ? sample : nullptr;
+  p.sample_step = sample_step;
+  p.sample_step_bias = sample_step_bias;
   const int tiles = p.num_m * p.num_n * p.splits;
   if (grid > tiles) grid = tiles;
   if (grid < 1) grid = 1;

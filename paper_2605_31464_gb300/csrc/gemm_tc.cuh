@@ -23,6 +23,7 @@
 #pragma once
 
 #include "ptx.cuh"
+#include "sampling.cuh"
 
 namespace gf {
 
@@ -39,14 +40,13 @@ struct GemmArgs {
   // SWAP + kStoreF32 only: per output row b, atomicMax of argmax_key(value, column) over the tile
   // (the greedy arg max of a logits row; the lowest column wins ties)
   unsigned long long* argmax_keys;
+  // with argmax_keys: when `sample` is set, the key is taken over the perturbed score
+  // l * (1/T) + G (Gumbel-max draw, sampling.cuh) of token t = *sample_step + sample_step_bias
+  // (t = sample_step_bias when sample_step is null); output column b is sampled row b
+  const SampleParams* sample;
+  const int32_t* sample_step;
+  int sample_step_bias;
 };
-
-// Orders (value, index) pairs by value, then by lower index: larger key = better.
-__device__ __forceinline__ unsigned long long argmax_key(float v, int idx) {
-  const uint32_t u = __float_as_uint(v);
-  const uint32_t ord = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
-  return ((unsigned long long)ord << 32) | (0xFFFFFFFFu - (uint32_t)idx);
-}
 
 template <int BN, bool SWAP = false>
 struct GemmCfg {
@@ -323,8 +323,24 @@ __global__ void __launch_bounds__(192, 1)
               // transpose-reduce the warp's 32 rows x 32 columns: after five halvings lane l holds
               // the best key of column c + l over this warp's rows
               unsigned long long k[32];
+              if (p.sample) {
+                const SampleParams sp = *p.sample;
+                const int t = (p.sample_step ? *p.sample_step : 0) + p.sample_step_bias;
 #pragma unroll
-              for (int i = 0; i < 32; ++i) k[i] = row_ok ? argmax_key(__uint_as_float(r[i]), row) : 0ull;
+                for (int q = 0; q < 8; ++q) {
+                  // one Philox block serves the four rows c + 4q .. c + 4q + 3 (r / 4 shared)
+                  uint64_t w[4];
+                  philox4x64_10((uint64_t)row, (uint64_t)t, (uint64_t)((c >> 2) + q), 0ull, sp.seed, 0ull, w);
+#pragma unroll
+                  for (int j = 0; j < 4; ++j) {
+                    const float z = fmaf(__uint_as_float(r[4 * q + j]), sp.inv_temp, gumbel_from_word(w[j]));
+                    k[4 * q + j] = row_ok ? argmax_key(z, row) : 0ull;
+                  }
+                }
+              } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i) k[i] = row_ok ? argmax_key(__uint_as_float(r[i]), row) : 0ull;
+              }
 #pragma unroll
               for (int o = 16; o >= 1; o >>= 1) {
                 const bool upper = (lane & o) != 0;

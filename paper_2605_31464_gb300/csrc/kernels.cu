@@ -153,15 +153,16 @@ cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, 
                     ldy);
 }
 
-__global__ void last_rows_kernel(const int32_t* offsets, int B, int32_t* row_idx) {
+__global__ void last_rows_kernel(const int32_t* offsets, int B, int32_t* row_idx, int repeats) {
   pdl_trigger();
   pdl_wait();
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b < B) row_idx[b] = offsets[b + 1] - 1;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < B * repeats) row_idx[i] = offsets[i / repeats + 1] - 1;
 }
-cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s) {
-  if (B <= 0) return cudaSuccess;
-  return launch_pdl(last_rows_kernel, dim3((B + 255) / 256), dim3(256), 0, s, offsets, B, row_idx);
+cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s, int repeats) {
+  if (B <= 0 || repeats <= 0) return cudaSuccess;
+  return launch_pdl(last_rows_kernel, dim3((B * repeats + 255) / 256), dim3(256), 0, s, offsets, B, row_idx,
+                    repeats);
 }
 
 // ------------------------------------------------------------------ RoPE + KV write
@@ -327,6 +328,123 @@ cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t
   if (B <= 0) return cudaSuccess;
   return launch_pdl(argmax_kernel, dim3(B), dim3(1024), 0, s, logits, ld, V, out, out2, out2_stride, step, col_base,
                     col_limit);
+}
+
+// ------------------------------------------------------------------ temperature sampling
+// One block per row: the largest argmax_key of the Gumbel-perturbed scores (sampling.cuh).
+__global__ void sample_kernel(const float* logits, int64_t ld, int V, SampleParams sp_val, const SampleParams* sp_dev,
+                              const int32_t* step, int step_bias, int32_t* out, int32_t* out2, int64_t out2_stride,
+                              int col_base, int col_limit) {
+  pdl_trigger();
+  pdl_wait();
+  const SampleParams sp = sp_dev ? *sp_dev : sp_val;
+  const int s = step ? *step : 0;
+  const int t = s + step_bias;
+  const int b = blockIdx.x;
+  const float* row = logits + (int64_t)b * ld;
+  unsigned long long best = 0ull;
+  for (int v = threadIdx.x; v < V; v += blockDim.x) {
+    const unsigned long long k = argmax_key(sample_score(row[v], sp, t, b, v), v);
+    best = k > best ? k : best;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+    best = other > best ? other : best;
+  }
+  __shared__ unsigned long long sk[32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (lane == 0) sk[warp] = best;
+  __syncthreads();
+  if (warp == 0) {
+    best = lane < (int)(blockDim.x >> 5) ? sk[lane] : 0ull;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long other = __shfl_xor_sync(0xffffffffu, best, o);
+      best = other > best ? other : best;
+    }
+    if (lane == 0) {
+      const int id = best ? (int)(0xFFFFFFFFu - (uint32_t)(best & 0xFFFFFFFFull)) : 0;
+      out[b] = id;
+      if (out2) {
+        const int col = col_base + s;
+        if (col < col_limit) out2[(int64_t)b * out2_stride + col] = id;
+      }
+    }
+  }
+}
+cudaError_t launch_sample(const float* logits, int64_t ld, int B, int V, SampleParams sp, const SampleParams* sp_dev,
+                          const int32_t* step, int step_bias, int32_t* out, int32_t* out2, int64_t out2_stride,
+                          int col_base, int col_limit, cudaStream_t s) {
+  if (B <= 0) return cudaSuccess;
+  return launch_pdl(sample_kernel, dim3(B), dim3(1024), 0, s, logits, ld, V, sp, sp_dev, step, step_bias, out, out2,
+                    out2_stride, col_base, col_limit);
+}
+
+// One thread per (item, k) of p and per item of conf: mean and population standard deviation
+// over the item's R consecutive rows.
+__global__ void repeat_stats_kernel(const float* p, const float* conf, int B, int R, int K, float* p_mean,
+                                    float* p_std, float* conf_mean, float* conf_std) {
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= B * (K + 1)) return;
+  const bool is_p = i < B * K;
+  const int b = is_p ? i / K : i - B * K;
+  const int k = is_p ? i % K : 0;
+  const float* x = is_p ? p + (int64_t)b * R * K + k : conf + (int64_t)b * R;
+  const int stride = is_p ? K : 1;
+  float sum = 0.f;
+  for (int j = 0; j < R; ++j) sum += x[(int64_t)j * stride];
+  const float mean = sum / (float)R;
+  float ss = 0.f;
+  for (int j = 0; j < R; ++j) {
+    const float d = x[(int64_t)j * stride] - mean;
+    ss += d * d;
+  }
+  const float sd = sqrtf(ss / (float)R);
+  if (is_p) {
+    if (p_mean) p_mean[i] = mean;
+    if (p_std) p_std[i] = sd;
+  } else {
+    if (conf_mean) conf_mean[b] = mean;
+    if (conf_std) conf_std[b] = sd;
+  }
+}
+cudaError_t launch_repeat_stats(const float* p, const float* conf, int B, int R, int K, float* p_mean, float* p_std,
+                                float* conf_mean, float* conf_std, cudaStream_t s) {
+  if (B <= 0 || R <= 0) return cudaSuccess;
+  const int n = B * (K + 1);
+  return launch_pdl(repeat_stats_kernel, dim3((n + 255) / 256), dim3(256), 0, s, p, conf, B, R, K, p_mean, p_std,
+                    conf_mean, conf_std);
+}
+
+// ------------------------------------------------------------------ forked sequences
+// Block (job, layer): the job's source page of this layer is copied, K rows then the transposed V rows.
+__global__ void fork_pages_kernel(bf16* k_cache, bf16* v_cache, const int4* jobs, int64_t page_elems,
+                                  int64_t layer_elems, int32_t* seq_len) {
+  pdl_trigger();
+  pdl_wait();
+  const int4 j = jobs[blockIdx.x];
+  if (blockIdx.y == 0 && threadIdx.x == 0) seq_len[j.y] = seq_len[j.x];
+  if (j.z < 0) return;
+  const int64_t src = (int64_t)blockIdx.y * layer_elems + (int64_t)j.z * page_elems;
+  const int64_t dst = (int64_t)blockIdx.y * layer_elems + (int64_t)j.w * page_elems;
+  const int64_t n16 = page_elems * (int64_t)sizeof(bf16) / 16;
+  const uint4* ks = reinterpret_cast<const uint4*>(k_cache + src);
+  const uint4* vs = reinterpret_cast<const uint4*>(v_cache + src);
+  uint4* kd = reinterpret_cast<uint4*>(k_cache + dst);
+  uint4* vd = reinterpret_cast<uint4*>(v_cache + dst);
+  for (int64_t i = threadIdx.x; i < n16; i += blockDim.x) {
+    kd[i] = ks[i];
+    vd[i] = vs[i];
+  }
+}
+cudaError_t launch_fork_pages(bf16* k_cache, bf16* v_cache, const int4* jobs, int n_jobs, int layers,
+                              int64_t page_elems, int64_t layer_elems, int32_t* seq_len, cudaStream_t s) {
+  if (n_jobs <= 0) return cudaSuccess;
+  return launch_pdl(fork_pages_kernel, dim3(n_jobs, layers), dim3(256), 0, s, k_cache, v_cache, jobs, page_elems,
+                    layer_elems, seq_len);
 }
 
 // ------------------------------------------------------------------ verdict (Sec. 2.1)

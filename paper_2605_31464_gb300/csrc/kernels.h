@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "sampling.cuh"
+
 namespace gf {
 
 using bf16 = __nv_bfloat16;
@@ -40,9 +42,13 @@ int gemm_smem_bytes(int bn);
 // kStoreF32, kAtomicF32 and kSwiGLU only.
 // argmax_keys (swap + kStoreF32 only): atomicMax per output row of the packed (value, column)
 // key of its largest element (see gemm_tc.cuh); the array must start at zero.
+// sample (device pointer, with argmax_keys): the keys rank the Gumbel-perturbed scores of token
+// t = *sample_step + sample_step_bias instead of the logits (temperature sampling, sampling.cuh).
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
-                        int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr);
+                        int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr,
+                        const SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
+                        int sample_step_bias = 0);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {
@@ -116,10 +122,25 @@ cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab
                          cudaStream_t s);
 cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
                            float eps, bf16* y, int64_t ldy, cudaStream_t s);
-cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s);
+// row_idx[b * repeats + j] = offsets[b + 1] - 1 for j < repeats (the last prompt row, once per repeat).
+cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s, int repeats = 1);
 cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,
                           int64_t out2_stride, cudaStream_t s, const int32_t* step = nullptr, int col_base = 0,
                           int col_limit = 1 << 30);
+// Temperature sampling of B rows of logits (Gumbel-max, sampling.cuh): out[b] = the draw of token
+// t = (*step if step) + step_bias for row b, with the parameters *sp_dev (or sp when sp_dev is null);
+// optionally also out2[b*stride + col], col = col_base (+ *step), when col < col_limit.
+cudaError_t launch_sample(const float* logits, int64_t ld, int B, int V, SampleParams sp, const SampleParams* sp_dev,
+                          const int32_t* step, int step_bias, int32_t* out, int32_t* out2, int64_t out2_stride,
+                          int col_base, int col_limit, cudaStream_t s);
+// Mean and population standard deviation over the R repeats of each of B items:
+// p [B*R][K] -> p_mean/p_std [B][K]; conf [B*R] -> conf_mean/conf_std [B] (any output may be null).
+cudaError_t launch_repeat_stats(const float* p, const float* conf, int B, int R, int K, float* p_mean, float* p_std,
+                                float* conf_mean, float* conf_std, cudaStream_t s);
+// Forked sequences: for each job (src slot, dst slot, src page, dst page) copy the page's K and V
+// rows of every layer when src page >= 0, and set seq_len[dst slot] = seq_len[src slot].
+cudaError_t launch_fork_pages(bf16* k_cache, bf16* v_cache, const int4* jobs, int n_jobs, int layers,
+                              int64_t page_elems, int64_t layer_elems, int32_t* seq_len, cudaStream_t s);
 cudaError_t launch_verdict(const float* logits, int64_t ld, int B, const int32_t* ids, int K, float tau, float* p,
                            float* conf, int32_t* arg, uint8_t* defer, cudaStream_t s);
 cudaError_t launch_set_seq_len(const int32_t* offsets, const int32_t* slots, int B, int32_t* seq_len,

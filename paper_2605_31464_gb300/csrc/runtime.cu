@@ -207,6 +207,7 @@ struct gf_model {
   int tok_stride = 0;
   int32_t* ctl = nullptr;  // [0]: device decode-step counter
   unsigned long long* keys = nullptr;  // [B_max] fused greedy arg max keys (kept at zero between uses)
+  gf::SampleParams* samp = nullptr;    // sampling parameters of the running sampled forecast
   // one CUDA graph per batch size for the decode step of gf_forecast_batch
   cudaStream_t cap_stream = nullptr;
   std::map<int, cudaGraphExec_t> graphs;
@@ -320,7 +321,8 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
 // keys: ask the LM-head GEMM to fuse the greedy arg max (*fused tells whether it could).
 int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
          cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0, unsigned long long* keys = nullptr,
-         bool* fused = nullptr) {
+         bool* fused = nullptr, const gf::SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
+         int sample_bias = 0) {
   if (M <= 0) return GF_OK;
   int bn, splits;
   bool swap;
@@ -341,7 +343,7 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
   if (fused) *fused = use_keys;
   if (swap)
     CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true,
-                       use_keys ? keys : nullptr));
+                       use_keys ? keys : nullptr, sample, sample_step, sample_bias));
   else
     CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
   m->launches += 1;
@@ -596,7 +598,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
 // the step can be captured once in a CUDA graph and replayed.
 int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float* logits_dst, int32_t* next_dst,
                 int32_t* tokens_col, int64_t tokens_stride, cudaStream_t s, int32_t* step = nullptr,
-                bool capturing = false) {
+                bool capturing = false, bool sampled = false) {
   CU(gf::launch_embed(ids, B, m->embed, m->vocab, m->d, m->dres, m->err, s));
   m->launches++;
   CU(cudaMemsetAsync(m->dqkv, 0, (size_t)B * m->qkv_dim * sizeof(float), s));
@@ -668,8 +670,9 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
   m->launches++;
   float* lg = logits_dst ? logits_dst : m->logits;
   bool fused = false;
+  // sampled: token t = *step + 1 of each row is drawn (temperature sampling, sampling.cuh)
   TRY(gemm(m, m->dxn, B, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, true, 0, 0,
-           next_dst ? m->keys : nullptr, &fused));
+           next_dst ? m->keys : nullptr, &fused, sampled ? m->samp : nullptr, step, 1));
   if (next_dst && fused) {
     // greedy tokens from the LM head's fused arg max; advances the sequences and the step counter
     CU(gf::launch_finish_step(m->keys, B, next_dst, tokens_col, tokens_stride, step, step ? 1 : 0,
@@ -677,7 +680,10 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     m->launches++;
   } else {
     if (next_dst) {
-      if (step)
+      if (sampled)
+        CU(gf::launch_sample(lg, m->vocab, B, m->vocab, gf::SampleParams{}, m->samp, step, 1, next_dst, tokens_col,
+                             tokens_stride, 1, step ? (int)tokens_stride : (1 << 30), s));
+      else if (step)
         CU(gf::launch_argmax(lg, m->vocab, B, m->vocab, next_dst, tokens_col, tokens_stride, s, step, 1,
                              (int)tokens_stride));
       else
@@ -695,8 +701,9 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
 // The decode step of gf_forecast_batch for a batch of B sequences whose
 // handles are in m->handles, captured once as a CUDA graph: ids and tokens
 // come from m->next, logits go to m->logits, generated tokens to m->tok_hist.
-int decode_graph(gf_model* m, int B, const int32_t* h, cudaGraphExec_t* out) {
-  auto it = m->graphs.find(B);
+int decode_graph(gf_model* m, int B, const int32_t* h, cudaGraphExec_t* out, bool sampled = false) {
+  const int key = B | (sampled ? 1 << 20 : 0);
+  auto it = m->graphs.find(key);
   if (it != m->graphs.end()) {
     *out = it->second;
     return GF_OK;
@@ -707,7 +714,7 @@ int decode_graph(gf_model* m, int B, const int32_t* h, cudaGraphExec_t* out) {
   const int64_t launches = m->launches;
   CU(cudaStreamBeginCapture(m->cap_stream, cudaStreamCaptureModeThreadLocal));
   int rc = decode_impl(m, B, h, m->next, m->logits, m->next, m->tok_hist, m->tok_stride, m->cap_stream, m->ctl,
-                       true);
+                       true, sampled);
   cudaGraph_t g = nullptr;
   const cudaError_t e = cudaStreamEndCapture(m->cap_stream, &g);
   m->prof_mask = mask;
@@ -726,7 +733,7 @@ int decode_graph(gf_model* m, int B, const int32_t* h, cudaGraphExec_t* out) {
     for (auto& kv : m->graphs) cudaGraphExecDestroy(kv.second);
     m->graphs.clear();
   }
-  m->graphs[B] = exec;
+  m->graphs[key] = exec;
   *out = exec;
   return GF_OK;
 }
@@ -756,20 +763,111 @@ int prepare_decode(gf_model* m, int B, const int32_t* h, cudaStream_t s) {
 
 }  // namespace
 
+// Validates a forecast call and assembles its prompts (incumbent ++ candidate) into m->prompt_ids.
+// poff receives the prompt offsets; the device copy sits at m->fcall + 2 (B + 1).
+int assemble_prompts(gf_model* m, int B, const int32_t* inc_ids, const int32_t* inc_offsets, const int32_t* cand_ids,
+                     const int32_t* cand_offsets, int n_decode, const int32_t* verdict_ids, int K, float tau,
+                     std::vector<int32_t>& poff, cudaStream_t s) {
+  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
+  if (!(tau >= 0.f && tau <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
+  if (n_decode < 0) return fail(GF_EINVAL, "n_decode < 0");
+  for (int k = 0; k < K; ++k)
+    if (verdict_ids[k] < 0 || verdict_ids[k] >= m->vocab) return fail(GF_EINVAL, "verdict id %d >= vocab", verdict_ids[k]);
+  if (inc_offsets[0] != 0 || cand_offsets[0] != 0) return fail(GF_EINVAL, "offsets must start at 0");
+  poff.assign(B + 1, 0);
+  for (int b = 0; b < B; ++b) {
+    const int ni = inc_offsets[b + 1] - inc_offsets[b], nc = cand_offsets[b + 1] - cand_offsets[b];
+    if (ni < 0 || nc < 0 || ni + nc < 1) return fail(GF_EINVAL, "item %d: bad lengths %d + %d", b, ni, nc);
+    if ((ni > 0 && !inc_ids) || (nc > 0 && !cand_ids)) return fail(GF_EINVAL, "null ids");
+    poff[b + 1] = poff[b] + ni + nc;
+  }
+  if (poff[B] > m->T_max) return fail(GF_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
+  std::vector<int32_t> desc;
+  desc.insert(desc.end(), inc_offsets, inc_offsets + B + 1);
+  desc.insert(desc.end(), cand_offsets, cand_offsets + B + 1);
+  desc.insert(desc.end(), poff.begin(), poff.end());
+  TRY(upload(m->staging, m->fcall, desc.data(), desc.size() * sizeof(int32_t), s));
+  CU(gf::launch_build_prompts(inc_ids, m->fcall, cand_ids, m->fcall + B + 1, m->fcall + 2 * (B + 1), B, poff[B],
+                              m->prompt_ids, s));
+  m->launches++;
+  return GF_OK;
+}
+
+// Repeats of prefilled sequences: row b * R + j is h[b] for j = 0 and otherwise a new slot whose
+// block table shares h[b]'s full 64-token pages (copy-free) and owns a fresh copy of its partial
+// last page plus the pages of n_decode more tokens.  jobs receives (src slot, dst slot, src page,
+// dst page) per fork for launch_fork_pages (pages -1: nothing to copy).  On failure every slot of
+// rows and h is released.
+int fork_sequences(gf_model* m, int B, int R, const int32_t* h, int n_decode, std::vector<int32_t>& rows,
+                   std::vector<int32_t>& jobs) {
+  std::vector<std::pair<int, int>> unused;
+  for (int b = 0; b < B; ++b) rows[(size_t)b * R] = h[b];
+  int rc = GF_OK;
+  for (int b = 0; b < B && rc == GF_OK; ++b) {
+    const int len = m->h_len[h[b]], full = len / 64;
+    for (int j = 1; j < R && rc == GF_OK; ++j) {
+      if (m->free_slots.empty()) {
+        rc = fail(GF_ECAPACITY, "no free sequence slots");
+        break;
+      }
+      const int slot = m->free_slots.back();
+      m->free_slots.pop_back();
+      m->live[slot] = 1;
+      m->h_len[slot] = len;
+      rows[(size_t)b * R + j] = slot;
+      share_pages(m, slot, h[b], full, &unused);
+      rc = alloc_pages(m, slot, full, (len + n_decode + 63) / 64 - full, &unused);
+      const bool partial = len % 64 != 0;
+      jobs.insert(jobs.end(), {h[b], slot, partial ? m->h_bt[(int64_t)h[b] * m->max_pages + full] : -1,
+                               partial ? m->h_bt[(int64_t)slot * m->max_pages + full] : -1});
+    }
+  }
+  if (rc != GF_OK) {
+    for (int r = 0; r < B * R; ++r)
+      if (rows[r] >= 0) release_slot(m, rows[r]);
+    for (int b = 0; b < B; ++b) rows[(size_t)b * R] = -1;
+  }
+  return rc;
+}
+
+// Token 0 of the B x R sampled rows: the final norm of each prompt's last position (once per
+// repeat), the LM head into lg and the draw (into m->next and column 0 of m->tok_hist).  The
+// prompt offsets are the ones assemble_prompts left on the device.
+int sampled_head(gf_model* m, int B, int R, float* lg, cudaStream_t s) {
+  const int BR = B * R;
+  CU(gf::launch_last_rows(m->fcall + 2 * (B + 1), B, m->last_idx, s, R));
+  CU(gf::launch_rmsnorm(m->resid, m->d, m->last_idx, BR, m->d, m->final_norm, m->cfg.rms_eps, m->dxn, m->d, s));
+  m->launches += 2;
+  bool fused = false;
+  TRY(gemm(m, m->dxn, BR, m->d, m->head, m->vocab, lg, m->vocab, gf::kStoreF32, s, false, 0, 0, m->keys, &fused,
+           m->samp, nullptr, 0));
+  if (fused)
+    CU(gf::launch_finish_step(m->keys, BR, m->next, m->tok_hist, m->tok_stride, nullptr, 0, 1 << 30, nullptr,
+                              nullptr, s));
+  else
+    CU(gf::launch_sample(lg, m->vocab, BR, m->vocab, gf::SampleParams{}, m->samp, nullptr, 0, m->next, m->tok_hist,
+                         m->tok_stride, 0, 1 << 30, s));
+  m->launches++;
+  return GF_OK;
+}
+
 // The part of a forecast after the prefill: n_decode greedy steps (the first eager, the rest one
 // replayed CUDA graph), the verdict on the final logits, and the release of the sequences.
 int decode_verdict_release(gf_model* m, int B, std::vector<int32_t>& h, int n_decode, const int32_t* verdict_ids,
                            int K, float tau, float* p, float* conf, int32_t* verdict_arg, uint8_t* defer,
-                           int32_t* tokens, float* final_logits, float* lg, cudaStream_t s) {
+                           int32_t* tokens, float* final_logits, float* lg, cudaStream_t s,
+                           bool sampled = false) {
   int rc = upload(m->staging, m->handles, h.data(), (size_t)B * sizeof(int32_t), s);
   if (rc == GF_OK && n_decode > 0) {
     lg = m->logits;
     if (cudaMemsetAsync(m->ctl, 0, sizeof(int32_t), s) != cudaSuccess) rc = fail(GF_ECUDA, "memset failed");
     // the first step runs eagerly (it also configures the kernels); the rest replay one captured graph
-    if (rc == GF_OK) rc = decode_impl(m, B, h.data(), m->next, m->logits, m->next, m->tok_hist, m->tok_stride, s, m->ctl);
+    if (rc == GF_OK)
+      rc = decode_impl(m, B, h.data(), m->next, m->logits, m->next, m->tok_hist, m->tok_stride, s, m->ctl, false,
+                       sampled);
     if (rc == GF_OK && n_decode > 1) {
       cudaGraphExec_t exec = nullptr;
-      rc = decode_graph(m, B, h.data(), &exec);
+      rc = decode_graph(m, B, h.data(), &exec, sampled);
       // algorithmic bytes of the replayed steps: every weight once per step, the cached K/V each
       // sequence reads, and the new K/V rows written
       double bytes = 0;
@@ -965,6 +1063,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->tok_hist, Bm * m->tok_stride);
   if (!rc) rc = dalloc(m, &m->ctl, 4);
   if (!rc) rc = dalloc(m, &m->keys, Bm);
+  if (!rc) rc = dalloc(m, &m->samp, 1);
   if (rc) return bail(rc);
 
   // ---- pack weights
@@ -1048,6 +1147,18 @@ int gf_release(gf_model* m, int32_t B, const int32_t* seq_handles) {
   return GF_OK;
 }
 
+int gf_sample_tokens(int32_t B, const float* logits, int64_t ld, int32_t V, uint64_t seed, int32_t token_index,
+                     float temperature, int32_t* out_ids, void* stream) {
+  if (B < 0 || V < 1 || ld < V || token_index < 0) return fail(GF_EINVAL, "bad shape");
+  if (!(temperature > 0.f) || !std::isfinite(temperature)) return fail(GF_EINVAL, "temperature must be > 0");
+  if (B == 0) return GF_OK;
+  if (!logits || !out_ids) return fail(GF_EINVAL, "null argument");
+  const gf::SampleParams sp{(unsigned long long)seed, 1.0f / temperature, 0};
+  CU(gf::launch_sample(logits, ld, B, V, sp, nullptr, nullptr, token_index, out_ids, nullptr, 0, 0, 0,
+                       reinterpret_cast<cudaStream_t>(stream)));
+  return GF_OK;
+}
+
 int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdict_ids, int32_t K, float tau,
                float* p, float* conf, int32_t* verdict_arg, uint8_t* defer, void* stream) {
   if (B < 0 || !logits || !verdict_ids || !p || !conf || !verdict_arg || !defer)
@@ -1068,29 +1179,9 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
   if (!m || !inc_offsets || !cand_offsets || !verdict_ids || !p || !conf || !verdict_arg || !defer)
     return fail(GF_EINVAL, "null argument");
   if (B < 1 || B > m->B_max) return fail(GF_EINVAL, "batch %d outside 1..%d", B, m->B_max);
-  if (K < 1 || K > 8) return fail(GF_EINVAL, "K = %d outside 1..8", K);
-  if (!(tau >= 0.f && tau <= 1.f)) return fail(GF_EINVAL, "tau outside [0, 1]");
-  if (n_decode < 0) return fail(GF_EINVAL, "n_decode < 0");
-  for (int k = 0; k < K; ++k)
-    if (verdict_ids[k] < 0 || verdict_ids[k] >= m->vocab) return fail(GF_EINVAL, "verdict id %d >= vocab", verdict_ids[k]);
-  if (inc_offsets[0] != 0 || cand_offsets[0] != 0) return fail(GF_EINVAL, "offsets must start at 0");
-  std::vector<int32_t> poff(B + 1, 0);
-  for (int b = 0; b < B; ++b) {
-    const int ni = inc_offsets[b + 1] - inc_offsets[b], nc = cand_offsets[b + 1] - cand_offsets[b];
-    if (ni < 0 || nc < 0 || ni + nc < 1) return fail(GF_EINVAL, "item %d: bad lengths %d + %d", b, ni, nc);
-    if ((ni > 0 && !inc_ids) || (nc > 0 && !cand_ids)) return fail(GF_EINVAL, "null ids");
-    poff[b + 1] = poff[b] + ni + nc;
-  }
-  if (poff[B] > m->T_max) return fail(GF_ECAPACITY, "prompt tokens exceed max_prefill_tokens");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  std::vector<int32_t> desc;
-  desc.insert(desc.end(), inc_offsets, inc_offsets + B + 1);
-  desc.insert(desc.end(), cand_offsets, cand_offsets + B + 1);
-  desc.insert(desc.end(), poff.begin(), poff.end());
-  TRY(upload(m->staging, m->fcall, desc.data(), desc.size() * sizeof(int32_t), s));
-  CU(gf::launch_build_prompts(inc_ids, m->fcall, cand_ids, m->fcall + B + 1, m->fcall + 2 * (B + 1), B, poff[B],
-                              m->prompt_ids, s));
-  m->launches++;
+  std::vector<int32_t> poff;
+  TRY(assemble_prompts(m, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, K, tau, poff, s));
   std::vector<int32_t> h(B);
   float* lg = (n_decode == 0 && final_logits) ? final_logits : m->logits;
   // tok_hist[b, s] is the input of decode step s: the arg max of the logits before it
@@ -1098,6 +1189,58 @@ int gf_forecast_batch(gf_model* m, int32_t B, const int32_t* inc_ids, const int3
                    m->tok_stride));
   return decode_verdict_release(m, B, h, n_decode, verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens,
                                 final_logits, lg, s);
+}
+
+int gf_forecast_batch_sampled(gf_model* m, int32_t B, const int32_t* inc_ids, const int32_t* inc_offsets,
+                              const int32_t* cand_ids, const int32_t* cand_offsets, int32_t n_decode,
+                              int32_t repeats, float temperature, uint64_t seed, const int32_t* verdict_ids,
+                              int32_t K, float tau, float* p, float* conf, int32_t* verdict_arg, uint8_t* defer,
+                              float* p_mean, float* p_std, float* conf_mean, float* conf_std, int32_t* tokens,
+                              float* final_logits, void* stream) {
+  if (!m || !inc_offsets || !cand_offsets || !verdict_ids || !p || !conf || !verdict_arg || !defer)
+    return fail(GF_EINVAL, "null argument");
+  if (repeats < 1) return fail(GF_EINVAL, "repeats = %d < 1", repeats);
+  if (!(temperature > 0.f) || !std::isfinite(temperature)) return fail(GF_EINVAL, "temperature must be > 0");
+  if (B < 1 || (int64_t)B * repeats > m->B_max)
+    return fail(GF_EINVAL, "batch %d x %d repeats outside 1..%d rows", B, repeats, m->B_max);
+  const int R = repeats, BR = B * R;
+  if ((int)m->free_slots.size() < BR) return fail(GF_ECAPACITY, "no free sequence slots");
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  std::vector<int32_t> poff;
+  TRY(assemble_prompts(m, B, inc_ids, inc_offsets, cand_ids, cand_offsets, n_decode, verdict_ids, K, tau, poff, s));
+  // each prompt is prefilled once; its repeats are forks that share its full KV pages
+  std::vector<int32_t> h(B);
+  TRY(prefill_impl(m, B, m->prompt_ids, poff.data(), n_decode, h.data(), nullptr, nullptr, s, nullptr, 0, 0, -1,
+                   false));
+  std::vector<int32_t> rows(BR, -1);
+  std::vector<int32_t> jobs;
+  int rc = fork_sequences(m, B, R, h.data(), n_decode, rows, jobs);
+  if (rc == GF_OK) rc = upload_block_table(m, s);
+  if (rc == GF_OK && !jobs.empty()) rc = upload(m->staging, m->call, jobs.data(), jobs.size() * sizeof(int32_t), s);
+  if (rc == GF_OK) {
+    const int64_t page_elems = (int64_t)m->nkv * 64 * m->hd;
+    if (gf::launch_fork_pages(m->k_cache, m->v_cache, reinterpret_cast<const int4*>(m->call), (int)jobs.size() / 4,
+                              m->L, page_elems, m->num_pages * page_elems, m->seq_len, s) != cudaSuccess)
+      rc = fail(GF_ECUDA, "fork launch failed");
+    m->launches++;
+  }
+  const gf::SampleParams sp{(unsigned long long)seed, 1.0f / temperature, 0};
+  if (rc == GF_OK) rc = upload(m->staging, m->samp, &sp, sizeof(sp), s);
+  // token 0 of every row from its prompt's last position: final norm, LM head and the draw
+  float* lg = (n_decode == 0 && final_logits) ? final_logits : m->logits;
+  if (rc == GF_OK) rc = sampled_head(m, B, R, lg, s);
+  if (rc != GF_OK) {
+    for (int r = 0; r < BR; ++r)
+      if (rows[r] >= 0) release_slot(m, rows[r]);
+    return rc;
+  }
+  TRY(decode_verdict_release(m, BR, rows, n_decode, verdict_ids, K, tau, p, conf, verdict_arg, defer, tokens,
+                             final_logits, lg, s, true));
+  if (p_mean || p_std || conf_mean || conf_std) {
+    CU(gf::launch_repeat_stats(p, conf, B, R, K, p_mean, p_std, conf_mean, conf_std, s));
+    m->launches++;
+  }
+  return GF_OK;
 }
 
 int gf_forecast_batch_shared(gf_model* m, int32_t B, const int32_t* prefix_ids, int32_t prefix_len,

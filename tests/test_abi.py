@@ -77,3 +77,20 @@ def test_null_model_calls_fail_cleanly(lib):
     with pytest.raises(gf.GfError):
         gf.gf_device_status(None, None)
     assert gf.gf_launch_count(None) == 0
+
+
+def test_sampling_argument_validation_needs_no_gpu(lib):
+    dummy = ctypes.c_void_p(16)
+    for T, t, V, ld in [(0.0, 0, 8, 8), (float("nan"), 0, 8, 8), (float("inf"), 0, 8, 8), (1.0, -1, 8, 8),
+                        (1.0, 0, 8, 4), (1.0, 0, 0, 8)]:
+        with pytest.raises(gf.GfError) as e:
+            gf.gf_sample_tokens(2, dummy, ld, V, 0, t, T, dummy, None)
+        assert e.value.code == gf.GF_EINVAL
+    off = np.array([0, 1], dtype=np.int32)
+    vid = np.array([10, 11], dtype=np.int32)
+    with pytest.raises(gf.GfError) as e:
+        gf.gf_forecast_batch_sampled(None, 1, dummy, off.ctypes.data_as(ctypes.c_void_p), dummy,
+                                     off.ctypes.data_as(ctypes.c_void_p), 4, 3, 1.0, 0,
+                                     vid.ctypes.data_as(ctypes.c_void_p), 2, 0.8, dummy, dummy, dummy, dummy, None,
+                                     None, None, None, None, None, None)
+    assert e.value.code == gf.GF_EINVAL
