@@ -36,6 +36,9 @@ static cudaError_t dispatch_mode(const CUtensorMap& tmA, const CUtensorMap& tmB,
     case kAtomicF32: return launch_one<BN, kAtomicF32, false>(tmA, tmB, p, grid, s);
     case kStoreBF16: return launch_one<BN, kStoreBF16, false>(tmA, tmB, p, grid, s);
     case kSwiGLU: return launch_one<BN, kSwiGLU, false>(tmA, tmB, p, grid, s);
+    case kRopeQKV:
+      if constexpr (BN >= 128) return launch_one<BN, kRopeQKV, false>(tmA, tmB, p, grid, s);
+      return cudaErrorInvalidValue;
     default: return cudaErrorInvalidValue;
   }
 }
@@ -54,11 +57,12 @@ static cudaError_t dispatch_swap(const CUtensorMap& tmA, const CUtensorMap& tmB,
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
                         bool swap, unsigned long long* argmax_keys, const SampleParams* sample,
-                        const int32_t* sample_step, int sample_step_bias) {
+                        const int32_t* sample_step, int sample_step_bias, const RopeEpilogue* rope) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0) return cudaErrorInvalidValue;
   if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
   if (swap && (M % 32 != 0 || N > bn)) return cudaErrorInvalidValue;
+  if (mode == kRopeQKV && (swap || !rope || bn < 128 || N % 128 != 0 || splits > 1)) return cudaErrorInvalidValue;
   GemmArgs p;
   p.M = M;
   p.N = N;
@@ -85,6 +89,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   p.sample = p.argmax_keys ? sample : nullptr;
   p.sample_step = sample_step;
   p.sample_step_bias = sample_step_bias;
+  if (rope) p.rope = *rope;
   const int tiles = p.num_m * p.num_n * p.splits;
   if (grid > tiles) grid = tiles;
   if (grid < 1) grid = 1;

@@ -12,6 +12,11 @@
 //   kSwiGLU     B rows are interleaved in blocks of 16 (16 gate rows, then
 //               the 16 matching up rows); the output is bf16(silu(gate) * up)
 //               with N/2 columns.
+//   kRopeQKV    prefill QKV projection: the columns are n_q query, n_kv key
+//               and n_kv value heads of 128; query and key heads are rotated
+//               (RoPE at each row's position) and, with the values, rounded
+//               to bf16 and written straight to the rotated-query buffer and
+//               the paged K / transposed-V cache (no fp32 QKV round trip).
 // The kernel is persistent: gridDim.x CTAs walk the tile list (grouped along
 // M so that concurrently running CTAs share A and B tiles in L2).
 //
@@ -27,7 +32,21 @@
 
 namespace gf {
 
-enum GemmMode { kStoreF32 = 0, kAddF32 = 1, kAtomicF32 = 2, kStoreBF16 = 3, kSwiGLU = 4 };
+enum GemmMode { kStoreF32 = 0, kAddF32 = 1, kAtomicF32 = 2, kStoreBF16 = 3, kSwiGLU = 4, kRopeQKV = 5 };
+
+// Destination of the kRopeQKV epilogue (head_dim 128).  Row t of the GEMM is token t of the
+// packed prompts, at sequence slot row_map[t].x and position row_map[t].y.
+struct RopeEpilogue {
+  const int2* row_map;
+  const float2* rope_cs;        // [position][64] (cos, sin) of position * theta^(-2i/128)
+  __nv_bfloat16* q_out;         // [T][n_q * 128]
+  int64_t ldq;
+  __nv_bfloat16* k_cache;       // rows of 128: [layer][page][n_kv][64 tokens]
+  __nv_bfloat16* v_cache;       // transposed pages: [layer][page][n_kv][128][64 tokens]
+  const int32_t* block_table;   // [slot][max_pages]
+  int max_pages, n_q, n_kv;
+  int64_t layer_row0;           // first K-cache row of this layer
+};
 
 struct GemmArgs {
   int M, N, K;
@@ -46,6 +65,7 @@ struct GemmArgs {
   const SampleParams* sample;
   const int32_t* sample_step;
   int sample_step_bias;
+  RopeEpilogue rope;  // kRopeQKV only
 };
 
 template <int BN, bool SWAP = false>
@@ -354,6 +374,57 @@ __global__ void __launch_bounds__(192, 1)
               }
               const int bb = c + lane;
               if (bb < p.N && k[0] != 0ull) atomicMax(p.argmax_keys + bb, k[0]);
+            }
+          }
+        }
+      } else if (MODE == kRopeQKV) {
+        // each 128-column block of the tile is one head; RoPE pairs columns i and i + 64
+        const RopeEpilogue& e = p.rope;
+        int2 rm = make_int2(0, 0);
+        if (row_ok) rm = e.row_map[row];
+        const int page = row_ok ? e.block_table[(int64_t)rm.x * e.max_pages + (rm.y >> 6)] : 0;
+        const int in_page = rm.y & 63;
+        const float4* cs4 = reinterpret_cast<const float4*>(e.rope_cs + (int64_t)rm.y * 64);
+#pragma unroll 1
+        for (int hh = 0; hh < BN / 128; ++hh) {
+          const int head = n_blk * (BN / 128) + hh;
+          if (head * 128 >= p.N) break;  // uniform across the CTA
+#pragma unroll 1
+          for (int c = 0; c < 64; c += 32) {
+            uint32_t lo[32], hi[32];
+            tmem_ld32(taddr + hh * 128 + c, lo);
+            tmem_ld32(taddr + hh * 128 + c + 64, hi);
+            tmem_ld_wait();
+            if (!row_ok) continue;
+            if (head < e.n_q + e.n_kv) {
+              uint32_t y0[16], y1[16];
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const float4 r = cs4[(c >> 1) + j];  // (cos, sin) of pairs c + 2j and c + 2j + 1
+                const float a0 = __uint_as_float(lo[2 * j]), b0 = __uint_as_float(hi[2 * j]);
+                const float a1 = __uint_as_float(lo[2 * j + 1]), b1 = __uint_as_float(hi[2 * j + 1]);
+                y0[j] = pack_bf16(a0 * r.x - b0 * r.y, a1 * r.z - b1 * r.w);
+                y1[j] = pack_bf16(b0 * r.x + a0 * r.y, b1 * r.z + a1 * r.w);
+              }
+              __nv_bfloat16* dst =
+                  head < e.n_q ? e.q_out + (int64_t)row * e.ldq + head * 128
+                               : e.k_cache + (e.layer_row0 + ((int64_t)page * e.n_kv + (head - e.n_q)) * 64 + in_page) * 128;
+              uint4* d0 = reinterpret_cast<uint4*>(dst + c);
+              uint4* d1 = reinterpret_cast<uint4*>(dst + c + 64);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) {
+                d0[q] = make_uint4(y0[4 * q], y0[4 * q + 1], y0[4 * q + 2], y0[4 * q + 3]);
+                d1[q] = make_uint4(y1[4 * q], y1[4 * q + 1], y1[4 * q + 2], y1[4 * q + 3]);
+              }
+            } else {
+              // values: [hd][64 tokens] per page, so lanes (consecutive tokens) write adjacent elements
+              const int g = head - e.n_q - e.n_kv;
+              __nv_bfloat16* dst = e.v_cache + e.layer_row0 * 128 + ((int64_t)page * e.n_kv + g) * 128 * 64 + in_page;
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                dst[(int64_t)(c + i) * 64] = __float2bfloat16(__uint_as_float(lo[i]));
+                dst[(int64_t)(c + 64 + i) * 64] = __float2bfloat16(__uint_as_float(hi[i]));
+              }
             }
           }
         }

@@ -243,6 +243,25 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
   }
 }
 
+__global__ void token_map_kernel(const int32_t* offsets, const int32_t* slots, const int32_t* past, int B, int T,
+                                 int2* map) {
+  pdl_trigger();
+  pdl_wait();
+  const int t = blockIdx.x * blockDim.x + threadIdx.x;
+  if (t >= T) return;
+  int lo = 0, hi = B - 1;  // item with offsets[item] <= t < offsets[item+1]
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (offsets[mid] <= t) lo = mid; else hi = mid - 1;
+  }
+  map[t] = make_int2(slots[lo], t - offsets[lo] + (past ? past[lo] : 0));
+}
+cudaError_t launch_token_map(const int32_t* offsets, const int32_t* slots, const int32_t* past, int B, int T,
+                             int2* map, cudaStream_t s) {
+  if (T <= 0) return cudaSuccess;
+  return launch_pdl(token_map_kernel, dim3((T + 255) / 256), dim3(256), 0, s, offsets, slots, past, B, T, map);
+}
+
 cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s) {
   if (a.T <= 0) return cudaSuccess;
   return launch_pdl(rope_kv_kernel, dim3(a.T), dim3(256), 0, s, a);

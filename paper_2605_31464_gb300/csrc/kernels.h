@@ -11,6 +11,7 @@
 namespace gf {
 
 using bf16 = __nv_bfloat16;
+struct RopeEpilogue;  // gemm_tc.cuh
 
 // Launch with programmatic stream serialization: the kernel may begin while the
 // previous kernel of the stream finishes; it must call pdl_wait() (ptx.cuh)
@@ -48,7 +49,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
                         int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr,
                         const SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
-                        int sample_step_bias = 0);
+                        int sample_step_bias = 0, const RopeEpilogue* rope = nullptr);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {
@@ -117,6 +118,9 @@ struct RopeKvArgs {
   int zero_after;             // write zeros back into qkv after reading (split-K accumulators)
 };
 cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s);
+// map[t] = (slot of the prompt holding packed token t, its position) for t < T.
+cudaError_t launch_token_map(const int32_t* offsets, const int32_t* slots, const int32_t* past, int B, int T,
+                             int2* map, cudaStream_t s);
 
 cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab, int d, float* out, int* err,
                          cudaStream_t s);

@@ -158,6 +158,7 @@ struct gf_model {
   float* resid = nullptr;
   bf16* xn = nullptr;
   float* qkv = nullptr;
+  int2* row_map = nullptr;  // prefill token -> (slot, position)
   bf16* q = nullptr;
   bf16* attn = nullptr;
   bf16* act = nullptr;
@@ -284,7 +285,7 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
   const int num_m = (M + 127) / 128;
   *splits = 1;
   *swap = false;
-  if (M <= 128 && N % 32 == 0 && (mode == gf::kStoreF32 || mode == gf::kAtomicF32 || mode == gf::kSwiGLU)) {
+  if (M <= 128 && N % 32 == 0 && (mode == gf::kStoreF32 || mode == gf::kAtomicF32 || mode == gf::kSwiGLU) ) {
     *swap = true;
     *bn = M <= 32 ? 32 : (M <= 64 ? 64 : 128);
     if (mode == gf::kAtomicF32) {
@@ -297,7 +298,7 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
     }
     return;
   }
-  if (mode == gf::kSwiGLU) {
+  if (mode == gf::kSwiGLU || mode == gf::kRopeQKV) {
     *bn = num_m >= 4 ? 256 : 128;
     return;
   }
@@ -322,7 +323,7 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
 int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
          cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0, unsigned long long* keys = nullptr,
          bool* fused = nullptr, const gf::SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
-         int sample_bias = 0) {
+         int sample_bias = 0, const gf::RopeEpilogue* rope = nullptr) {
   if (M <= 0) return GF_OK;
   int bn, splits;
   bool swap;
@@ -336,7 +337,8 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
     TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, (uint32_t)bn, &tb));
   }
   const double na = n_alg ? n_alg : N, ka = k_alg ? k_alg : K;
-  const double out_bytes = (mode == gf::kSwiGLU ? na / 2 * 2 : na * (mode == gf::kStoreBF16 ? 2 : 4)) * M;
+  const double out_bytes =
+      (mode == gf::kSwiGLU ? na / 2 * 2 : na * (mode == gf::kStoreBF16 || mode == gf::kRopeQKV ? 2 : 4)) * M;
   ProfScope ps(m, s, decode ? GF_PROF_DECODE_GEMM : GF_PROF_PREFILL_GEMM, 2.0 * M * na * ka,
                na * ka * 2 + (double)M * ka * 2 + out_bytes * (mode == gf::kAddF32 || mode == gf::kAtomicF32 ? 2 : 1));
   const bool use_keys = keys && swap && mode == gf::kStoreF32;
@@ -345,7 +347,8 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
     CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true,
                        use_keys ? keys : nullptr, sample, sample_step, sample_bias));
   else
-    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s));
+    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, false, nullptr, nullptr,
+                       nullptr, 0, rope));
   m->launches += 1;
   return GF_OK;
 }
@@ -501,6 +504,23 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
 
   CU(gf::launch_embed(ids, (int)T, m->embed, m->vocab, m->d, m->resid, m->err, s));
   m->launches++;
+  // head_dim 128: RoPE and the KV-cache write are fused into the QKV GEMM's epilogue
+  const bool fused_rope = m->hd == 128;
+  gf::RopeEpilogue re{};
+  if (fused_rope) {
+    CU(gf::launch_token_map(d_off, d_slots, d_past, B, (int)T, m->row_map, s));
+    m->launches++;
+    re.row_map = m->row_map;
+    re.rope_cs = m->rope_cs;
+    re.q_out = m->q;
+    re.ldq = m->q_dim;
+    re.k_cache = m->k_cache;
+    re.v_cache = m->v_cache;
+    re.block_table = m->bt;
+    re.max_pages = m->max_pages;
+    re.n_q = m->nq;
+    re.n_kv = m->nkv;
+  }
   CUtensorMap tq;
   TRY(get_map(m, m->q, (uint64_t)m->q_dim, (uint64_t)T, 128, &tq));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)m->hd);
@@ -509,29 +529,35 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
     TRY(fire_captures(m, l, m->resid, offsets, B, false, s));
     CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.attn_norm, m->cfg.rms_eps, m->xn, m->d, s));
     m->launches++;
-    TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, m->qkv, m->qkv_dim, gf::kStoreF32, s, false));
-    gf::RopeKvArgs ra{};
-    ra.qkv = m->qkv;
-    ra.ldqkv = m->qkv_dim;
-    ra.q_out = m->q;
-    ra.ldq = m->q_dim;
-    ra.k_cache = m->k_cache;
-    ra.v_cache = m->v_cache;
-    ra.rope_cs = m->rope_cs;
-    ra.offsets = d_off;
-    ra.slots = d_slots;
-    ra.past = d_past;
-    ra.B = B;
-    ra.block_table = m->bt;
-    ra.max_pages = m->max_pages;
-    ra.T = (int)T;
-    ra.n_q = m->nq;
-    ra.n_kv = m->nkv;
-    ra.hd = m->hd;
-    ra.layer_row0 = layer_row0(m, l);
-    ra.zero_after = 0;
-    CU(gf::launch_rope_kv(ra, s));
-    m->launches++;
+    if (fused_rope) {
+      re.layer_row0 = layer_row0(m, l);
+      TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, nullptr, 0, gf::kRopeQKV, s, false, 0, 0, nullptr, nullptr,
+               nullptr, nullptr, 0, &re));
+    } else {
+      TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, m->qkv, m->qkv_dim, gf::kStoreF32, s, false));
+      gf::RopeKvArgs ra{};
+      ra.qkv = m->qkv;
+      ra.ldqkv = m->qkv_dim;
+      ra.q_out = m->q;
+      ra.ldq = m->q_dim;
+      ra.k_cache = m->k_cache;
+      ra.v_cache = m->v_cache;
+      ra.rope_cs = m->rope_cs;
+      ra.offsets = d_off;
+      ra.slots = d_slots;
+      ra.past = d_past;
+      ra.B = B;
+      ra.block_table = m->bt;
+      ra.max_pages = m->max_pages;
+      ra.T = (int)T;
+      ra.n_q = m->nq;
+      ra.n_kv = m->nkv;
+      ra.hd = m->hd;
+      ra.layer_row0 = layer_row0(m, l);
+      ra.zero_after = 0;
+      CU(gf::launch_rope_kv(ra, s));
+      m->launches++;
+    }
     gf::PrefillAttnArgs pa{};
     pa.items = d_items;
     pa.offsets = d_off;
@@ -1036,6 +1062,7 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->resid, T * d);
   if (!rc) rc = dalloc(m, &m->xn, T * d);
   if (!rc) rc = dalloc(m, &m->qkv, T * m->qkv_dim);
+  if (!rc) rc = dalloc(m, &m->row_map, T);
   if (!rc) rc = dalloc(m, &m->q, T * m->q_dim);
   if (!rc) rc = dalloc(m, &m->attn, T * m->q_dim);
   if (!rc) rc = dalloc(m, &m->act, T * m->ffn_pad);

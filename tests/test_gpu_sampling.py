@@ -202,3 +202,37 @@ def test_sampled_forecast_rejects_bad_arguments(tiny):
             _run_sampled(m, prompts, 2, kw["R"], kw["T"], 0)
         assert e.value.code == gf.GF_EINVAL
     assert m.free_pages() == free0
+
+
+@pytest.fixture(scope="module")
+def gqa_wide():
+    m = make_model(GQA, max_batch=128, max_seq=512, max_prefill_tokens=4096)
+    yield GQA, m, oracle.Weights(GQA)
+    m.close()
+
+
+def test_many_rows_use_the_wide_lm_head_tiles(gqa_wide):
+    # 4 items x 25 repeats = 100 rows: the LM-head draw runs on 128-column tiles with several
+    # 32-row chunks and a ragged last chunk; the oracle checks the prompt draw and one decode draw
+    shape, m, W = gqa_wide
+    prompts = _ragged_prompts(shape.vocab)
+    R, T, seed = 25, 1.0, 31337
+    out = _run_sampled(m, prompts, 2, R, T, seed)
+    m.status()
+    toks = out["tokens"].cpu().numpy()
+    lg = out["logits"].cpu().numpy()
+    prompt_logits = {}
+    for r in range(4 * R):
+        i = r // R
+        if i not in prompt_logits:
+            prompt_logits[i] = oracle.prefill(W, _prompt(*prompts, i))[0]
+        sc = smp.sample_scores(prompt_logits[i], T, smp.uniforms(seed, 0, r, shape.vocab))
+        assert _draw_agrees(int(toks[r, 0]), sc, ARGMAX_GAP), f"row {r} token 0"
+    for r in (0, 1, 27, 50, 77, 99):
+        ref = smp.forecast_sampled_one(W, _prompt(*prompts, r // R), 2, VIDS, TAU, seed, r, T, forced_tokens=toks[r])
+        sc = smp.sample_scores(ref["step_logits"][1], T, smp.uniforms(seed, 1, r, shape.vocab))
+        assert _draw_agrees(int(toks[r, 1]), sc, ARGMAX_GAP), f"row {r} token 1"
+        check_logits(lg[r], ref["step_logits"][-1], f"row {r} final logits")
+    # 25 draws from one prompt's distribution are not all the same token
+    for i in range(4):
+        assert len(set(toks[i * R:(i + 1) * R, 0].tolist())) > 1
