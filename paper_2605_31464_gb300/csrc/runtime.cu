@@ -478,15 +478,16 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   desc.insert(desc.end(), (size_t)B, past);
   const size_t items_at = desc.size() + (desc.size() & 1);  // int2 alignment
   desc.resize(items_at);
+  // attention work items: (prompt, pair of 128-row query tiles)
   std::vector<std::pair<int, int>> items;
   for (int b = 0; b < B; ++b) {
     const int len = offsets[b + 1] - offsets[b];
-    for (int qt = 0; qt < (len + 127) / 128; ++qt) items.push_back({b, qt});
+    for (int qt = 0; qt < (len + 255) / 256; ++qt) items.push_back({b, qt});
   }
   std::stable_sort(items.begin(), items.end(), [&](const std::pair<int, int>& x, const std::pair<int, int>& y) {
     auto cost = [&](const std::pair<int, int>& it) {
       const int len = offsets[it.first + 1] - offsets[it.first];
-      return past + std::min(it.second * 128 + 128, len);
+      return past + std::min(it.second * 256 + 256, len);
     };
     return cost(x) > cost(y);
   });
