@@ -8,6 +8,11 @@
 // double-buffered; warp w takes keys 16w..16w+15 of each page.
 // Each CTA writes an unnormalised partial (running max, running sum, sum of
 // p.v) for its chunk; attn_combine merges the chunks of a sequence.
+// In the model's decode step the kernel also does the RoPE pass (see
+// DecodeAttnArgs::qkv): the queries are rotated by every CTA for its group,
+// and the new key (rotated) and value are written into the cache by the CTA
+// whose chunk holds the new token, before its TMA reads that page; the merge
+// kernel then zeroes the rows of the split-K sums that were read.
 #include <mutex>
 
 #include "gf.h"
@@ -49,7 +54,8 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int kvh = blockIdx.y;
   const int b = blockIdx.z;
   const int slot = a.handles ? a.handles[b] : b;
-  const int ctx = min(a.seq_len[slot] + a.ctx_bias, a.max_ctx);
+  const int pos = a.seq_len[slot];  // the new token's position (fused step)
+  const int ctx = min(pos + a.ctx_bias, a.max_ctx);
   const int k0 = split * a.chunk;
   if (k0 >= ctx) return;
   const int k1 = min(k0 + a.chunk, ctx);
@@ -70,20 +76,77 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
     tma_load_2d(sV + buf * C::PAGE_BYTES, &tmV, &bar[buf], 0, (int)(a.layer_vrow0 + pg * HD));
   };
 
+  const bool fused = a.qkv != nullptr;
+  const bool writes_kv = fused && k1 == ctx;  // this chunk holds the new token
+  // The page holding the new token is read only after this CTA has written the token into it: when
+  // that page is among the first STAGES, its copy waits for the block-wide barrier below; later
+  // pages are issued after the per-page barrier of the main loop anyway.
+  const int first_copies = min(C::STAGES, n_pages);
+  const bool defer_last = writes_kv && n_pages <= C::STAGES;
   if (threadIdx.x == 0) {
     for (int i = 0; i < C::STAGES; ++i) mbar_init(&bar[i], 1);
     fence_mbar_init();
     fence_async_smem();
-    for (int i = 0; i < C::STAGES && i < n_pages; ++i) issue(i);
+    for (int i = 0; i < first_copies - (defer_last ? 1 : 0); ++i) issue(i);
   }
-  // Q rows of this group (zero rows beyond G), 16-byte chunks, swizzled like TMA.
-  for (int c = threadIdx.x; c < 16 * (HD / 8); c += blockDim.x) {
-    const int r = c / (HD / 8), ch = c % (HD / 8);
-    uint4 v = make_uint4(0, 0, 0, 0);
-    if (r < G) v = *reinterpret_cast<const uint4*>(a.q + (int64_t)b * a.ldq + (kvh * G + r) * HD + ch * 8);
-    *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (16 * 128) + sw128(r, ch & 7)) = v;
+  if (fused) {
+    // rotated queries of this group as bf16, swizzled like TMA; rows G..15 are zero.  Each thread
+    // handles up to four (row, pair) items, all loads first.
+    const float* row = a.qkv + (int64_t)b * a.ldqkv;
+    const float2* cs = a.rope_cs + (int64_t)pos * (HD / 2);
+    constexpr int kItems = 16 * (HD / 2) / 128;  // (row, pair) items per thread over all 16 rows
+    float x0[kItems], x1[kItems];
+    float2 t[kItems];
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) {
+      const int c = threadIdx.x + u * 128, r = c / (HD / 2), i = c % (HD / 2);
+      x0[u] = x1[u] = 0.f;
+      t[u] = make_float2(0.f, 0.f);
+      if (r < G) {
+        x0[u] = row[(kvh * G + r) * HD + i];
+        x1[u] = row[(kvh * G + r) * HD + i + HD / 2];
+        t[u] = cs[i];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) {
+      const int c = threadIdx.x + u * 128, r = c / (HD / 2), i = c % (HD / 2);
+      const float y0 = x0[u] * t[u].x - x1[u] * t[u].y;
+      const float y1 = x1[u] * t[u].x + x0[u] * t[u].y;
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const int col = i + hh * (HD / 2);
+        *reinterpret_cast<bf16*>(sQ + (col >> 6) * (16 * 128) + sw128(r, (col & 63) >> 3) + (col & 7) * 2) =
+            __float2bfloat16(hh ? y1 : y0);
+      }
+    }
+    if (writes_kv) {
+      const int page = pages[pos >> 6], in_page = pos & 63;
+      const float* kr = row + (a.n_q + kvh) * HD;
+      const float* vr = row + (a.n_q + a.n_kv + kvh) * HD;
+      bf16* kd = a.k_cache + (a.layer_row0 + ((int64_t)page * a.n_kv + kvh) * 64 + in_page) * HD;
+      bf16* vd = a.v_cache + a.layer_vrow0 * 64 + ((int64_t)page * a.n_kv + kvh) * HD * 64 + in_page;
+      const float2* cs2 = a.rope_cs + (int64_t)pos * (HD / 2);
+      for (int i = threadIdx.x; i < HD / 2; i += blockDim.x) {
+        const float x0 = kr[i], x1 = kr[i + HD / 2];
+        const float2 t = cs2[i];
+        kd[i] = __float2bfloat16(x0 * t.x - x1 * t.y);
+        kd[i + HD / 2] = __float2bfloat16(x1 * t.x + x0 * t.y);
+      }
+      for (int d = threadIdx.x; d < HD; d += blockDim.x) vd[(int64_t)d * 64] = __float2bfloat16(vr[d]);
+      fence_async_global();  // the page's TMA read (after a block-wide barrier) must see these writes
+    }
+  } else {
+    // Q rows of this group (zero rows beyond G), 16-byte chunks, swizzled like TMA.
+    for (int c = threadIdx.x; c < 16 * (HD / 8); c += blockDim.x) {
+      const int r = c / (HD / 8), ch = c % (HD / 8);
+      uint4 v = make_uint4(0, 0, 0, 0);
+      if (r < G) v = *reinterpret_cast<const uint4*>(a.q + (int64_t)b * a.ldq + (kvh * G + r) * HD + ch * 8);
+      *reinterpret_cast<uint4*>(sQ + (ch >> 3) * (16 * 128) + sw128(r, ch & 7)) = v;
+    }
   }
   __syncthreads();
+  if (defer_last && threadIdx.x == 0) issue(n_pages - 1);
 
   uint32_t qa[HD / 16][4];
   {
@@ -264,6 +327,18 @@ __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
       O += a.part_o[((base + s) * 16 + r) * HD + d] * f;
     }
     a.out[(int64_t)b * a.ldo + h * HD + d] = __float2bfloat16(L > 0.f ? O / L : 0.f);
+  }
+  if (a.qkv) {
+    // fused step: every attention CTA has read its queries and the new key and value; zero the
+    // split-K sums of this query head (and of the group's key and value heads) for the next step
+    float* row = a.qkv + (int64_t)b * a.ldqkv;
+    for (int d = threadIdx.x; d < HD; d += blockDim.x) {
+      row[h * HD + d] = 0.f;
+      if (r == 0) {
+        row[(a.n_q + kvh) * HD + d] = 0.f;
+        row[(a.n_q + a.n_kv + kvh) * HD + d] = 0.f;
+      }
+    }
   }
 }
 

@@ -90,6 +90,15 @@ struct DecodeAttnArgs {
   int64_t ldo;
   float scale_log2;
   int* err;
+  // Fused decode step (qkv != nullptr; q is then unused): the queries and the new token's key and
+  // value are read from the fp32 split-K sums of the QKV projection and rotated at position
+  // seq_len[slot], the key and value written into the cache, and the merge kernel sets the rows of
+  // qkv that were read back to zero for the next step's split-K sums.
+  float* qkv;                 // [B, ldqkv]: n_q query heads | n_kv key heads | n_kv value heads
+  int64_t ldqkv;
+  const float2* rope_cs;      // [position][hd/2]
+  bf16* k_cache;              // rows of hd: [layer][page][n_kv][64 tokens]
+  bf16* v_cache;              // [layer][page][n_kv][hd][64 tokens]
 };
 cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a,
                                int B, cudaStream_t s);

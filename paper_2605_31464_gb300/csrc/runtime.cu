@@ -168,7 +168,6 @@ struct gf_model {
   float* dres = nullptr;
   bf16* dxn = nullptr;
   float* dqkv = nullptr;
-  bf16* dq = nullptr;
   bf16* dattn = nullptr;
   bf16* dact = nullptr;
   float *part_o = nullptr, *part_ml = nullptr;
@@ -635,31 +634,10 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     if (!capturing) TRY(fire_captures(m, l, m->dres, nullptr, B, true, s));
     CU(gf::launch_rmsnorm(m->dres, m->d, nullptr, B, m->d, W.attn_norm, m->cfg.rms_eps, m->dxn, m->d, s));
     m->launches++;
+    // split-K sums of q | k | v; the attention kernel rotates them, writes the new key and value
+    // into the cache and zeroes these rows again
     TRY(gemm(m, m->dxn, B, m->d, W.qkv, m->qkv_dim, m->dqkv, m->qkv_dim, gf::kAtomicF32, s, true));
-    gf::RopeKvArgs ra{};
-    ra.qkv = m->dqkv;
-    ra.ldqkv = m->qkv_dim;
-    ra.q_out = m->dq;
-    ra.ldq = m->q_dim;
-    ra.k_cache = m->k_cache;
-    ra.v_cache = m->v_cache;
-    ra.rope_cs = m->rope_cs;
-    ra.offsets = nullptr;
-    ra.handles = m->handles;
-    ra.seq_len = m->seq_len;
-    ra.block_table = m->bt;
-    ra.max_pages = m->max_pages;
-    ra.T = B;
-    ra.n_q = m->nq;
-    ra.n_kv = m->nkv;
-    ra.hd = m->hd;
-    ra.layer_row0 = layer_row0(m, l);
-    ra.zero_after = 1;
-    CU(gf::launch_rope_kv(ra, s));
-    m->launches++;
     gf::DecodeAttnArgs da{};
-    da.q = m->dq;
-    da.ldq = m->q_dim;
     da.handles = m->handles;
     da.seq_len = m->seq_len;
     da.ctx_bias = 1;
@@ -678,6 +656,11 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     da.ldo = m->q_dim;
     da.scale_log2 = scale_log2;
     da.err = m->err;
+    da.qkv = m->dqkv;
+    da.ldqkv = m->qkv_dim;
+    da.rope_cs = m->rope_cs;
+    da.k_cache = m->k_cache;
+    da.v_cache = m->v_cache;
     {
       double ctx = 0;
       for (int b = 0; b < B; ++b) ctx += m->h_len[h[b]] + 1;
@@ -1073,7 +1056,6 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->dres, Bm * d);
   if (!rc) rc = dalloc(m, &m->dxn, Bm * d);
   if (!rc) rc = dalloc(m, &m->dqkv, Bm * m->qkv_dim);
-  if (!rc) rc = dalloc(m, &m->dq, Bm * m->q_dim);
   if (!rc) rc = dalloc(m, &m->dattn, Bm * m->q_dim);
   if (!rc) rc = dalloc(m, &m->dact, Bm * m->ffn_pad);
   if (!rc) rc = dalloc(m, &m->part_o, Bm * m->nkv * m->dec_max_splits * 16 * hd);
@@ -1557,6 +1539,10 @@ int gf_device_status(gf_model* m, void* stream) {
   int h = 0;
   CU(cudaMemcpy(&h, m->err, sizeof(int), cudaMemcpyDeviceToHost));
   CU(cudaMemset(m->err, 0, sizeof(int)));
+  if (h != 0) {
+    // a kernel that gave up may have left split-K sums behind
+    CU(cudaMemset(m->dqkv, 0, (size_t)m->B_max * m->qkv_dim * sizeof(float)));
+  }
   if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a device-side wait timed out");
   if (h == 1) return fail(GF_EINVAL, "a token id outside [0, vocab) reached the device");
   if (h != 0) return fail(GF_ECUDA, "device error word %d", h);
