@@ -92,7 +92,7 @@ def _prefill(a):
     ids_d = torch.from_numpy(ids).cuda()
     s = torch.cuda.current_stream()
     for r in range(a.repeat + 1):
-        if r == 1:
+        if r == min(1, a.repeat):  # with --repeat 0 the single run is timed (no warm-up)
             e0 = torch.cuda.Event(enable_timing=True)
             e0.record(s)
         h, _, _ = m.prefill(ids_d, off, want_logits=False)
@@ -134,7 +134,7 @@ def _forecast(a):
     inc_d, cand_d = torch.from_numpy(inc).cuda(), torch.from_numpy(cand).cuda()
     s = torch.cuda.current_stream()
     for r in range(a.repeat + 1):
-        if r == 1:
+        if r == min(1, a.repeat):  # with --repeat 0 the single run is timed (no warm-up)
             m.profile(1 << gf.GF_PROF_DECODE_STEPS)
             m.profile_read(gf.GF_PROF_DECODE_STEPS)
             e0 = torch.cuda.Event(enable_timing=True)
