@@ -218,3 +218,28 @@ def test_pool_exhaustion_and_bad_handles_are_reported():
     m.release(h)
     m.status()
     m.close()
+
+
+def test_more_than_128_sequences_use_the_wide_decode_tiles():
+    # 160 sequences: the decode GEMMs leave the few-rows (swapped) path, the greedy token comes from a
+    # separate arg-max kernel, and decode attention runs 160 x n_kv groups
+    m = make_model(GQA, max_batch=160, max_seq=256, max_prefill_tokens=160 * 48)
+    W = oracle.Weights(GQA)
+    try:
+        lens = [17 + (i * 7) % 31 for i in range(160)]  # 17..47 tokens
+        ids = synth.uniform_int(9, 3, sum(lens), 0, GQA.vocab - 1)
+        off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+        io = np.zeros(161, dtype=np.int32)  # no incumbent: every prompt is its candidate part
+        out = m.forecast_batch(_cuda_i32(np.zeros(1, dtype=np.int32)), io, _cuda_i32(ids), off, 4, (10, 11), 0.8,
+                               want_tokens=True, want_logits=True)
+        torch.cuda.synchronize()
+        m.status()
+        toks = out["tokens"].cpu().numpy()
+        lg = out["logits"].cpu().numpy()
+        for i in (0, 1, 63, 64, 127, 128, 129, 159):
+            ref = oracle.forecast_one(W, ids[off[i]:off[i + 1]], 4, (10, 11), 0.8, forced_tokens=toks[i])
+            check_logits(lg[i], ref["step_logits"][-1], f"final logits item {i}")
+            for t in range(4):
+                assert greedy_agrees(int(toks[i, t]), ref["step_logits"][t]), f"item {i} token {t}"
+    finally:
+        m.close()

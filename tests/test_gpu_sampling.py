@@ -236,3 +236,34 @@ def test_many_rows_use_the_wide_lm_head_tiles(gqa_wide):
     # 25 draws from one prompt's distribution are not all the same token
     for i in range(4):
         assert len(set(toks[i * R:(i + 1) * R, 0].tolist())) > 1
+
+
+@pytest.fixture(scope="module")
+def tiny_wide():
+    w = synth.workload("tiny")
+    m = make_model(w.model, max_batch=160, max_seq=512, max_prefill_tokens=4096)
+    yield w.model, m, oracle.Weights(w.model)
+    m.close()
+
+
+def test_more_than_128_rows_draw_outside_the_lm_head_gemm(tiny_wide):
+    # 4 items x 40 repeats = 160 rows: beyond the widest fused LM-head tile the logits are written out
+    # and a separate kernel draws every row, in the prompt step and inside the captured decode graph
+    shape, m, W = tiny_wide
+    prompts = _tiny_prompts()
+    R, T, seed, n_decode = 40, 1.0, 4242, 3
+    free0 = m.free_pages()
+    out = _run_sampled(m, prompts, n_decode, R, T, seed)
+    m.status()
+    assert m.free_pages() == free0
+    toks = out["tokens"].cpu().numpy()
+    lg = out["logits"].cpu().numpy()
+    for r in (0, 1, 39, 40, 77, 120, 159):
+        ref = smp.forecast_sampled_one(W, _prompt(*prompts, r // R), n_decode, VIDS, TAU, seed, r, T,
+                                       forced_tokens=toks[r])
+        for t in range(n_decode):
+            sc = smp.sample_scores(ref["step_logits"][t], T, smp.uniforms(seed, t, r, shape.vocab))
+            assert _draw_agrees(int(toks[r, t]), sc, ARGMAX_GAP), f"row {r} token {t}"
+        check_logits(lg[r], ref["step_logits"][-1], f"row {r} final logits")
+    for i in range(4):
+        assert len({tuple(toks[i * R + j]) for j in range(R)}) > 1
