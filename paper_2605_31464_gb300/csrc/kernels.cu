@@ -166,6 +166,8 @@ cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cu
 }
 
 // ------------------------------------------------------------------ RoPE + KV write
+// Prefill of models whose head_dim is not 128 (with 128 the QKV GEMM's epilogue does this, and
+// decode attention does it for the decode step).
 // One block per token.  q and k heads are rotated pairwise (i, i + hd/2) by
 // angle pos * theta^(-2i/hd) (cos/sin from the table), rounded to bf16 and
 // written to the rotated-query buffer or the key cache ([page][kv head][64
@@ -175,19 +177,13 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
   pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x;
-  int slot, pos;
-  if (a.offsets) {
-    int lo = 0, hi = a.B - 1;  // item with offsets[item] <= t < offsets[item+1]
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (a.offsets[mid] <= t) lo = mid; else hi = mid - 1;
-    }
-    slot = a.slots[lo];
-    pos = t - a.offsets[lo] + (a.past ? a.past[lo] : 0);
-  } else {
-    slot = a.handles[t];
-    pos = a.seq_len[slot];
+  int lo = 0, hi = a.B - 1;  // item with offsets[item] <= t < offsets[item+1]
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (a.offsets[mid] <= t) lo = mid; else hi = mid - 1;
   }
+  const int slot = a.slots[lo];
+  const int pos = t - a.offsets[lo] + (a.past ? a.past[lo] : 0);
   const int half = a.hd / 2;
   const int heads = a.n_q + 2 * a.n_kv;
   const int page = a.block_table[(int64_t)slot * a.max_pages + (pos >> 6)];
@@ -214,10 +210,6 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
       if (idx >= n) continue;
       const int h = idx / half, i = idx % half;
       const int c0 = h * a.hd + i;
-      if (a.zero_after) {
-        src[c0] = 0.f;
-        src[c0 + half] = 0.f;
-      }
       if (h < a.n_q + a.n_kv) {
         const float2 r = cs[i];
         const bf16 y0 = __float2bfloat16(x0[u] * r.x - x1[u] * r.y);

@@ -112,19 +112,15 @@ struct RopeKvArgs {
   bf16* k_cache;
   bf16* v_cache;
   const float2* rope_cs;      // [max_seq][hd/2] (cos, sin)
-  // prefill: offsets/slots (and past: cached positions before each prompt, or nullptr) describe the
-  // packed prompts; decode: offsets == nullptr
+  // the packed prompts: offsets/slots (and past: cached positions before each prompt, or nullptr)
   const int32_t* offsets;
   const int32_t* slots;
   const int32_t* past;
   int B;
-  const int32_t* handles;
-  const int32_t* seq_len;
   const int32_t* block_table;
   int max_pages;
   int T, n_q, n_kv, hd;
   int64_t layer_row0;
-  int zero_after;             // write zeros back into qkv after reading (split-K accumulators)
 };
 cudaError_t launch_rope_kv(const RopeKvArgs& a, cudaStream_t s);
 // map[t] = (slot of the prompt holding packed token t, its position) for t < T.

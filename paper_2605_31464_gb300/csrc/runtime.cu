@@ -554,7 +554,6 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
       ra.n_kv = m->nkv;
       ra.hd = m->hd;
       ra.layer_row0 = layer_row0(m, l);
-      ra.zero_after = 0;
       CU(gf::launch_rope_kv(ra, s));
       m->launches++;
     }
