@@ -57,7 +57,8 @@ static cudaError_t dispatch_swap(const CUtensorMap& tmA, const CUtensorMap& tmB,
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
                         bool swap, unsigned long long* argmax_keys, const SampleParams* sample,
-                        const int32_t* sample_step, int sample_step_bias, const RopeEpilogue* rope) {
+                        const int32_t* sample_step, int sample_step_bias, const RopeEpilogue* rope,
+                        const NormFold* norm) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0) return cudaErrorInvalidValue;
   if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
@@ -90,6 +91,22 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   p.sample_step = sample_step;
   p.sample_step_bias = sample_step_bias;
   if (rope) p.rope = *rope;
+  p.norm_out = nullptr;
+  p.norm_gain = nullptr;
+  p.norm_ss = nullptr;
+  p.ld_norm = 0;
+  p.row_ss = nullptr;
+  p.inv_d = 0.f;
+  p.eps = 0.f;
+  if (norm && !swap) {
+    p.norm_out = norm->out;
+    p.norm_gain = norm->gain;
+    p.norm_ss = norm->ss_out;
+    p.ld_norm = norm->ld_out;
+    p.row_ss = norm->ss_in;
+    p.inv_d = norm->inv_d;
+    p.eps = norm->eps;
+  }
   const int tiles = p.num_m * p.num_n * p.splits;
   if (grid > tiles) grid = tiles;
   if (grid < 1) grid = 1;

@@ -66,6 +66,17 @@ struct GemmArgs {
   const int32_t* sample_step;
   int sample_step_bias;
   RopeEpilogue rope;  // kRopeQKV only
+  // RMSNorm folded into the prefill GEMMs around it (non-swapped tiles only):
+  //  kAddF32 with norm_out: after the residual update also write norm_out = bf16(x_new * norm_gain[col])
+  //    and add the row's sum of x_new^2 over the tile's columns into norm_ss[row] (atomically);
+  //  kSwiGLU / kRopeQKV with row_ss: the accumulator row is scaled by rsqrt(row_ss[row] * inv_d + eps)
+  //    before the epilogue's arithmetic, so that A = bf16(x * gain) yields RMSNorm(x) * gain . W.
+  __nv_bfloat16* norm_out;
+  const float* norm_gain;
+  float* norm_ss;
+  int64_t ld_norm;
+  const float* row_ss;
+  float inv_d, eps;
 };
 
 template <int BN, bool SWAP = false>
@@ -385,6 +396,7 @@ __global__ void __launch_bounds__(192, 1)
         const int page = row_ok ? e.block_table[(int64_t)rm.x * e.max_pages + (rm.y >> 6)] : 0;
         const int in_page = rm.y & 63;
         const float4* cs4 = reinterpret_cast<const float4*>(e.rope_cs + (int64_t)rm.y * 64);
+        const float rs = (p.row_ss && row_ok) ? rsqrtf(p.row_ss[row] * p.inv_d + p.eps) : 1.f;
 #pragma unroll 1
         for (int hh = 0; hh < BN / 128; ++hh) {
           const int head = n_blk * (BN / 128) + hh;
@@ -396,6 +408,13 @@ __global__ void __launch_bounds__(192, 1)
             tmem_ld32(taddr + hh * 128 + c + 64, hi);
             tmem_ld_wait();
             if (!row_ok) continue;
+            if (rs != 1.f) {
+#pragma unroll
+              for (int i = 0; i < 32; ++i) {
+                lo[i] = __float_as_uint(__uint_as_float(lo[i]) * rs);
+                hi[i] = __float_as_uint(__uint_as_float(hi[i]) * rs);
+              }
+            }
             if (head < e.n_q + e.n_kv) {
               uint32_t y0[16], y1[16];
 #pragma unroll
@@ -430,6 +449,7 @@ __global__ void __launch_bounds__(192, 1)
         }
       } else if (MODE == kSwiGLU) {
         // each 32-column chunk holds 16 gate columns then the 16 matching up columns
+        const float rs = (p.row_ss && row_ok) ? rsqrtf(p.row_ss[row] * p.inv_d + p.eps) : 1.f;
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
@@ -440,8 +460,8 @@ __global__ void __launch_bounds__(192, 1)
             uint32_t o[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
-              const float g0 = __uint_as_float(r[2 * j]), g1 = __uint_as_float(r[2 * j + 1]);
-              const float u0 = __uint_as_float(r[16 + 2 * j]), u1 = __uint_as_float(r[16 + 2 * j + 1]);
+              const float g0 = __uint_as_float(r[2 * j]) * rs, g1 = __uint_as_float(r[2 * j + 1]) * rs;
+              const float u0 = __uint_as_float(r[16 + 2 * j]) * rs, u1 = __uint_as_float(r[16 + 2 * j + 1]) * rs;
               o[j] = pack_bf16(g0 / (1.0f + __expf(-g0)) * u0, g1 / (1.0f + __expf(-g1)) * u1);
             }
             uint4* dst = reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(p.out) + (int64_t)row * p.ldo +
@@ -450,6 +470,45 @@ __global__ void __launch_bounds__(192, 1)
             dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
           }
         }
+      } else if (MODE == kAddF32) {
+        float ss = 0.f;
+#pragma unroll 1
+        for (int c = 0; c < BN; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(taddr + c, r);
+          tmem_ld_wait();
+          const int col = n_blk * BN + c;
+          if (row_ok && col < p.N) {
+            float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + col);
+            float x[32];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const float4 o = dst[i];
+              x[4 * i] = o.x + __uint_as_float(r[4 * i]);
+              x[4 * i + 1] = o.y + __uint_as_float(r[4 * i + 1]);
+              x[4 * i + 2] = o.z + __uint_as_float(r[4 * i + 2]);
+              x[4 * i + 3] = o.w + __uint_as_float(r[4 * i + 3]);
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i) dst[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
+            if (p.norm_out) {
+              const float4* g4 = reinterpret_cast<const float4*>(p.norm_gain + col);
+              uint32_t pk[16];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) {
+                const float4 g = g4[i];
+                ss += x[4 * i] * x[4 * i] + x[4 * i + 1] * x[4 * i + 1] + x[4 * i + 2] * x[4 * i + 2] +
+                      x[4 * i + 3] * x[4 * i + 3];
+                pk[2 * i] = pack_bf16(x[4 * i] * g.x, x[4 * i + 1] * g.y);
+                pk[2 * i + 1] = pack_bf16(x[4 * i + 2] * g.z, x[4 * i + 3] * g.w);
+              }
+              uint4* nd = reinterpret_cast<uint4*>(p.norm_out + (int64_t)row * p.ld_norm + col);
+#pragma unroll
+              for (int q = 0; q < 4; ++q) nd[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+            }
+          }
+        }
+        if (p.norm_out && row_ok) atomicAdd(p.norm_ss + row, ss);
       } else {
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {

@@ -142,6 +142,47 @@ __global__ void __launch_bounds__(256) rmsnorm_warp_kernel(const float* x, int64
   }
 }
 
+// Folded RMSNorm (prefill): y[r, :] = bf16(x[r, :] * gain) and ss[r] = sum(x[r, :]^2); the GEMM that
+// reads y applies rsqrt(ss / d + eps) to its output rows.  One warp per row.
+__global__ void __launch_bounds__(256) norm_stats_kernel(const float* x, int rows, int d, const float* gain, bf16* y,
+                                                         float* ss_out) {
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x * (blockDim.x / 32) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (r >= rows) return;
+  const float4* xr = reinterpret_cast<const float4*>(x + (int64_t)r * d);
+  const float4* g4 = reinterpret_cast<const float4*>(gain);
+  uint2* yr = reinterpret_cast<uint2*>(y + (int64_t)r * d);
+  const int nv = d / 4;
+  float ss = 0.f;
+  for (int base = lane; base < nv; base += 8 * 32) {
+    float4 v[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) v[k] = base + k * 32 < nv ? xr[base + k * 32] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int i = base + k * 32;
+      ss += v[k].x * v[k].x + v[k].y * v[k].y + v[k].z * v[k].z + v[k].w * v[k].w;
+      if (i < nv) {
+        const float4 g = g4[i];
+        uint2 o;
+        o.x = pack_bf16(v[k].x * g.x, v[k].y * g.y);
+        o.y = pack_bf16(v[k].z * g.z, v[k].w * g.w);
+        yr[i] = o;
+      }
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+  if (lane == 0) ss_out[r] = ss;
+}
+cudaError_t launch_norm_stats(const float* x, int rows, int d, const float* gain, bf16* y, float* ss, cudaStream_t s) {
+  if (rows <= 0) return cudaSuccess;
+  if (d % 4) return cudaErrorInvalidValue;
+  return launch_pdl(norm_stats_kernel, dim3((rows + 7) / 8), dim3(256), 0, s, x, rows, d, gain, y, ss);
+}
+
 cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
                            float eps, bf16* y, int64_t ldy, cudaStream_t s) {
   if (rows <= 0) return cudaSuccess;
@@ -209,7 +250,6 @@ __global__ void rope_kv_kernel(const RopeKvArgs a) {
       const int idx = base + u * blockDim.x;
       if (idx >= n) continue;
       const int h = idx / half, i = idx % half;
-      const int c0 = h * a.hd + i;
       if (h < a.n_q + a.n_kv) {
         const float2 r = cs[i];
         const bf16 y0 = __float2bfloat16(x0[u] * r.x - x1[u] * r.y);

@@ -13,6 +13,18 @@ namespace gf {
 using bf16 = __nv_bfloat16;
 struct RopeEpilogue;  // gemm_tc.cuh
 
+// RMSNorm folded into prefill GEMMs (see GemmArgs in gemm_tc.cuh): a residual-update GEMM writes
+// out = bf16(x_new * gain) and adds sum(x_new^2) per row into ss_out; a consumer GEMM reading such an
+// out scales its accumulator row by rsqrt(ss_in[row] * inv_d + eps).
+struct NormFold {
+  bf16* out;
+  const float* gain;
+  float* ss_out;
+  int64_t ld_out;
+  const float* ss_in;
+  float inv_d, eps;
+};
+
 // Launch with programmatic stream serialization: the kernel may begin while the
 // previous kernel of the stream finishes; it must call pdl_wait() (ptx.cuh)
 // before using that kernel's results.
@@ -49,7 +61,8 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
                         int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr,
                         const SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
-                        int sample_step_bias = 0, const RopeEpilogue* rope = nullptr);
+                        int sample_step_bias = 0, const RopeEpilogue* rope = nullptr,
+                        const NormFold* norm = nullptr);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {
@@ -131,6 +144,8 @@ cudaError_t launch_embed(const int32_t* ids, int T, const bf16* table, int vocab
                          cudaStream_t s);
 cudaError_t launch_rmsnorm(const float* x, int64_t ldx, const int32_t* row_idx, int rows, int d, const float* gain,
                            float eps, bf16* y, int64_t ldy, cudaStream_t s);
+// The folded form (many rows): y = bf16(x * gain) un-normalised and ss[r] = sum(x[r, :]^2).
+cudaError_t launch_norm_stats(const float* x, int rows, int d, const float* gain, bf16* y, float* ss, cudaStream_t s);
 // row_idx[b * repeats + j] = offsets[b + 1] - 1 for j < repeats (the last prompt row, once per repeat).
 cudaError_t launch_last_rows(const int32_t* offsets, int B, int32_t* row_idx, cudaStream_t s, int repeats = 1);
 cudaError_t launch_argmax(const float* logits, int64_t ld, int B, int V, int32_t* out, int32_t* out2,

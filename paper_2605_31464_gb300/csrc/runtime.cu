@@ -159,6 +159,7 @@ struct gf_model {
   bf16* xn = nullptr;
   float* qkv = nullptr;
   int2* row_map = nullptr;  // prefill token -> (slot, position)
+  float *ss_attn = nullptr, *ss_ffn = nullptr;  // prefill row sums of squares for the folded RMSNorm
   bf16* q = nullptr;
   bf16* attn = nullptr;
   bf16* act = nullptr;
@@ -322,11 +323,17 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
 int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
          cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0, unsigned long long* keys = nullptr,
          bool* fused = nullptr, const gf::SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
-         int sample_bias = 0, const gf::RopeEpilogue* rope = nullptr) {
+         int sample_bias = 0, const gf::RopeEpilogue* rope = nullptr, const gf::NormFold* norm = nullptr) {
   if (M <= 0) return GF_OK;
   int bn, splits;
   bool swap;
   plan_gemm(m->sms, M, N, K, mode, &bn, &splits, &swap);
+  if (norm && swap) {
+    // the folded RMSNorm is applied by the row-major (non-swapped) epilogues only
+    swap = false;
+    bn = 128;
+    splits = 1;
+  }
   CUtensorMap ta, tb;
   if (swap) {
     TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, 128, &ta));
@@ -347,7 +354,7 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
                        use_keys ? keys : nullptr, sample, sample_step, sample_bias));
   else
     CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, false, nullptr, nullptr,
-                       nullptr, 0, rope));
+                       nullptr, 0, rope, norm));
   m->launches += 1;
   return GF_OK;
 }
@@ -524,15 +531,30 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   CUtensorMap tq;
   TRY(get_map(m, m->q, (uint64_t)m->q_dim, (uint64_t)T, 128, &tq));
   const float scale_log2 = 1.4426950408889634f / sqrtf((float)m->hd);
+  // With the fused RoPE path the two RMSNorms of a layer are folded into the GEMMs around them: the
+  // residual-update GEMMs write xn = bf16(x * gain) with per-row sums of squares, and the QKV and
+  // gate/up GEMMs scale their output rows by rsqrt(mean square + eps).
+  gf::NormFold to_qkv{}, to_gu{}, from_o{}, from_down{};
+  if (fused_rope) {
+    const float inv_d = 1.0f / (float)m->d;
+    to_qkv = gf::NormFold{nullptr, nullptr, nullptr, 0, m->ss_attn, inv_d, m->cfg.rms_eps};
+    to_gu = gf::NormFold{nullptr, nullptr, nullptr, 0, m->ss_ffn, inv_d, m->cfg.rms_eps};
+    from_o = gf::NormFold{m->xn, nullptr, m->ss_ffn, m->d, nullptr, 0.f, 0.f};
+    from_down = gf::NormFold{m->xn, nullptr, m->ss_attn, m->d, nullptr, 0.f, 0.f};
+    CU(gf::launch_norm_stats(m->resid, (int)T, m->d, m->layers[0].attn_norm, m->xn, m->ss_attn, s));
+    m->launches++;
+  }
   for (int l = 0; l < m->L; ++l) {
     const gf_model::Layer& W = m->layers[l];
     TRY(fire_captures(m, l, m->resid, offsets, B, false, s));
-    CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.attn_norm, m->cfg.rms_eps, m->xn, m->d, s));
-    m->launches++;
+    if (!fused_rope) {
+      CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.attn_norm, m->cfg.rms_eps, m->xn, m->d, s));
+      m->launches++;
+    }
     if (fused_rope) {
       re.layer_row0 = layer_row0(m, l);
       TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, nullptr, 0, gf::kRopeQKV, s, false, 0, 0, nullptr, nullptr,
-               nullptr, nullptr, 0, &re));
+               nullptr, nullptr, 0, &re, &to_qkv));
     } else {
       TRY(gemm(m, m->xn, (int)T, m->d, W.qkv, m->qkv_dim, m->qkv, m->qkv_dim, gf::kStoreF32, s, false));
       gf::RopeKvArgs ra{};
@@ -583,12 +605,29 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
       CU(gf::launch_attn_prefill(m->hd, tq, m->tm_k, m->tm_v, pa, (int)items.size(), s));
     }
     m->launches++;
-    TRY(gemm(m, m->attn, (int)T, m->q_dim, W.o, m->d, m->resid, m->d, gf::kAddF32, s, false));
-    CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.ffn_norm, m->cfg.rms_eps, m->xn, m->d, s));
-    m->launches++;
-    TRY(gemm(m, m->xn, (int)T, m->d, W.gu, 2 * m->ffn_pad, m->act, m->ffn_pad, gf::kSwiGLU, s, false,
-             2 * m->ffn));
-    TRY(gemm(m, m->act, (int)T, m->ffn_pad, W.down, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, m->ffn));
+    if (fused_rope) {
+      CU(cudaMemsetAsync(m->ss_ffn, 0, (size_t)T * sizeof(float), s));
+      from_o.gain = W.ffn_norm;
+      TRY(gemm(m, m->attn, (int)T, m->q_dim, W.o, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, 0, nullptr, nullptr,
+               nullptr, nullptr, 0, nullptr, &from_o));
+      TRY(gemm(m, m->xn, (int)T, m->d, W.gu, 2 * m->ffn_pad, m->act, m->ffn_pad, gf::kSwiGLU, s, false, 2 * m->ffn, 0,
+               nullptr, nullptr, nullptr, nullptr, 0, nullptr, &to_gu));
+      // the last layer's output goes to the final norm (on the last rows only), not to another QKV
+      const bool next = l + 1 < m->L;
+      if (next) {
+        CU(cudaMemsetAsync(m->ss_attn, 0, (size_t)T * sizeof(float), s));
+        from_down.gain = m->layers[l + 1].attn_norm;
+      }
+      TRY(gemm(m, m->act, (int)T, m->ffn_pad, W.down, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, m->ffn, nullptr,
+               nullptr, nullptr, nullptr, 0, nullptr, next ? &from_down : nullptr));
+    } else {
+      TRY(gemm(m, m->attn, (int)T, m->q_dim, W.o, m->d, m->resid, m->d, gf::kAddF32, s, false));
+      CU(gf::launch_rmsnorm(m->resid, m->d, nullptr, (int)T, m->d, W.ffn_norm, m->cfg.rms_eps, m->xn, m->d, s));
+      m->launches++;
+      TRY(gemm(m, m->xn, (int)T, m->d, W.gu, 2 * m->ffn_pad, m->act, m->ffn_pad, gf::kSwiGLU, s, false,
+               2 * m->ffn));
+      TRY(gemm(m, m->act, (int)T, m->ffn_pad, W.down, m->d, m->resid, m->d, gf::kAddF32, s, false, 0, m->ffn));
+    }
   }
   TRY(fire_captures(m, m->L, m->resid, offsets, B, false, s));
   if (!want_head) {
@@ -1046,6 +1085,8 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->xn, T * d);
   if (!rc) rc = dalloc(m, &m->qkv, T * m->qkv_dim);
   if (!rc) rc = dalloc(m, &m->row_map, T);
+  if (!rc) rc = dalloc(m, &m->ss_attn, T);
+  if (!rc) rc = dalloc(m, &m->ss_ffn, T);
   if (!rc) rc = dalloc(m, &m->q, T * m->q_dim);
   if (!rc) rc = dalloc(m, &m->attn, T * m->q_dim);
   if (!rc) rc = dalloc(m, &m->act, T * m->ffn_pad);
