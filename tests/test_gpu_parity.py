@@ -243,3 +243,19 @@ def test_more_than_128_sequences_use_the_wide_decode_tiles():
                 assert greedy_agrees(int(toks[i, t]), ref["step_logits"][t]), f"item {i} token {t}"
     finally:
         m.close()
+
+
+@pytest.mark.parametrize("T", [1, 50, 128, 129])
+def test_gqa_short_prefill_uses_row_major_tiles_for_the_folded_norm(gqa, T):
+    # at most 128 prompt tokens would put the SwiGLU GEMM on the swapped (few-rows) tiles; the folded
+    # RMSNorm keeps it on the row-major ones
+    m, W = gqa
+    ids = synth.uniform_int(6, T, T, 0, GQA.vocab - 1)
+    out = m.forecast_batch(_cuda_i32(np.zeros(1, np.int32)), [0, 0], _cuda_i32(ids), [0, T], 3, (10, 11), 0.8,
+                           want_tokens=True, want_logits=True)
+    torch.cuda.synchronize()
+    m.status()
+    toks = out["tokens"].cpu().numpy()
+    ref = oracle.forecast_one(W, ids, 3, (10, 11), 0.8, forced_tokens=toks[0])
+    check_logits(out["logits"][0].cpu().numpy(), ref["step_logits"][-1], f"T={T}")
+    assert greedy_agrees(int(toks[0, 0]), ref["step_logits"][0])
