@@ -49,7 +49,7 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
 // tensor maps (bf16, 128-byte swizzle) with boxes {64, 128} and {64, bn}.
 int gemm_num_stages(int bn);
 int gemm_smem_bytes(int bn);
-// group_m: M-blocks per raster group (0 = sized so a group's A tiles fill about 48 MiB of L2).
+// group_m: M-blocks per raster group (0 = sized so a group's A tiles fill about 28 MiB of L2).
 // swap: A holds the weights (M = output features, multiple of 32), B the activations
 // (N = rows <= bn, bn 32/64/128), and out is written transposed (out[n][m]); modes
 // kStoreF32, kAtomicF32 and kSwiGLU only.
