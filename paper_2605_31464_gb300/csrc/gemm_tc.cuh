@@ -471,23 +471,35 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       } else if (MODE == kAddF32) {
+        // the residual chunk of the next 32 columns is loaded while this chunk is added and stored
         float ss = 0.f;
+        float* res_row = reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + n_blk * BN;
+        const int ncols = min(BN, p.N - n_blk * BN);
+        float4 cur[8], nxt[8];
+        if (row_ok && ncols > 0) {
+#pragma unroll
+          for (int i = 0; i < 8; ++i) cur[i] = reinterpret_cast<const float4*>(res_row)[i];
+        }
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
           uint32_t r[32];
           tmem_ld32(taddr + c, r);
+          const bool have_next = row_ok && c + 32 < ncols;
+          if (have_next) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) nxt[i] = reinterpret_cast<const float4*>(res_row + c + 32)[i];
+          }
           tmem_ld_wait();
           const int col = n_blk * BN + c;
-          if (row_ok && col < p.N) {
-            float4* dst = reinterpret_cast<float4*>(reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + col);
+          if (row_ok && c < ncols) {
+            float4* dst = reinterpret_cast<float4*>(res_row + c);
             float x[32];
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-              const float4 o = dst[i];
-              x[4 * i] = o.x + __uint_as_float(r[4 * i]);
-              x[4 * i + 1] = o.y + __uint_as_float(r[4 * i + 1]);
-              x[4 * i + 2] = o.z + __uint_as_float(r[4 * i + 2]);
-              x[4 * i + 3] = o.w + __uint_as_float(r[4 * i + 3]);
+              x[4 * i] = cur[i].x + __uint_as_float(r[4 * i]);
+              x[4 * i + 1] = cur[i].y + __uint_as_float(r[4 * i + 1]);
+              x[4 * i + 2] = cur[i].z + __uint_as_float(r[4 * i + 2]);
+              x[4 * i + 3] = cur[i].w + __uint_as_float(r[4 * i + 3]);
             }
 #pragma unroll
             for (int i = 0; i < 8; ++i) dst[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
@@ -506,6 +518,10 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
               for (int q = 0; q < 4; ++q) nd[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
             }
+          }
+          if (have_next) {
+#pragma unroll
+            for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
           }
         }
         if (p.norm_out && row_ok) atomicAdd(p.norm_ss + row, ss);
