@@ -34,7 +34,7 @@ import synth  # noqa: E402
 # same kernel build, or None when no capture of this build exists.
 # 7b_prefill: dram__bytes_read + dram__bytes_write per launch, averaged over the
 # prefill GEMM launches of one forecast on this workload.
-NCU_TRAFFIC = {"7b_prefill": 19.95e9}
+NCU_TRAFFIC = {"7b_prefill": 18.66e9}
 
 
 def parse_args():
