@@ -365,7 +365,8 @@ def test_planted_mistakes_are_caught(monkeypatch, target, bad):
     failed = 0
     for pin in _pins():
         try:
-            pin()
+            with np.errstate(invalid="ignore"):  # a planted mask can leave a row with no key (NaN)
+                pin()
         except (AssertionError, FloatingPointError, ValueError, IndexError):
             failed += 1
     assert failed >= 1, f"no pin caught the planted mistake in {target}"
