@@ -33,8 +33,10 @@ import synth  # noqa: E402
 # DRAM bytes per launch of the dominant kernel, from an ncu capture of the
 # same kernel build, or None when no capture of this build exists.
 # 7b_prefill: dram__bytes_read + dram__bytes_write per launch, averaged over the
-# prefill GEMM launches of one forecast on this workload.
-NCU_TRAFFIC = {"7b_prefill": 18.66e9}
+# 113 prefill GEMM launches of one forecast (28 layers x 4 + the LM head),
+# captured on 4 x 6144 tokens with two layers and scaled by the 8x rows (the
+# traffic of these GEMMs grows in proportion to the rows).
+NCU_TRAFFIC = {"7b_prefill": 18.41e9}
 
 
 def parse_args():

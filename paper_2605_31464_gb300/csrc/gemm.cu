@@ -58,7 +58,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s, int group_m,
                         bool swap, unsigned long long* argmax_keys, const SampleParams* sample,
                         const int32_t* sample_step, int sample_step_bias, const RopeEpilogue* rope,
-                        const NormFold* norm) {
+                        const NormFold* norm, bool w_blocked) {
   if (M <= 0 || N <= 0) return cudaSuccess;
   if (K % 64 != 0) return cudaErrorInvalidValue;
   if (!swap && N % 32 != 0) return cudaErrorInvalidValue;
@@ -100,6 +100,7 @@ cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, i
   p.row_ss = nullptr;
   p.inv_d = 0.f;
   p.eps = 0.f;
+  p.w_blocked = w_blocked ? 1 : 0;
   if (norm && !swap) {
     p.norm_out = norm->out;
     p.norm_gain = norm->gain;

@@ -2,6 +2,10 @@
 //
 // A (activations) and B (weights, rows = output features) are K-major bf16 in
 // global memory, streamed by TMA into 128-byte-swizzled shared-memory stages.
+// The weights are either row-major [N][K] or, with w_blocked, stored in blocks
+// of 256 rows x 64 columns, [ceil(N/256)][K/64][256][64] (zero rows pad N), so
+// that every weight box a stage loads (up to 256 rows of one 64-column slice)
+// is one contiguous run of memory instead of rows K*2 bytes apart.
 // One thread issues tcgen05.mma (M=128, N=BN, K=16 per instruction) into a
 // double-buffered fp32 accumulator in tensor memory; four epilogue warps read
 // it back with tcgen05.ld and apply the fused epilogue:
@@ -77,6 +81,7 @@ struct GemmArgs {
   int64_t ld_norm;
   const float* row_ss;
   float inv_d, eps;
+  int w_blocked;  // weights in 256 x 64 blocks (see the top of this file)
 };
 
 template <int BN, bool SWAP = false>
@@ -92,6 +97,19 @@ struct GemmCfg {
   static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
   static constexpr int THREADS = 192;
 };
+
+// TMA coordinates of the weight box for k-block kb at weight row row0 (a multiple of the box
+// height, which divides 256).  Blocked weights are addressed as a 2D map of 64-element rows:
+// block (row0 / 256, kb) starts at row (row0 / 256 * kb_total + kb) * 256.
+__device__ __forceinline__ void weight_coords(const GemmArgs& p, int kb, int row0, int& x, int& y) {
+  if (p.w_blocked) {
+    x = 0;
+    y = ((row0 >> 8) * p.kb_total + kb) * 256 + (row0 & 255);
+  } else {
+    x = kb * 64;
+    y = row0;
+  }
+}
 
 __device__ __forceinline__ void gemm_tile_coords(const GemmArgs& p, int tile, int& m_blk, int& n_blk, int& split) {
   split = tile % p.splits;
@@ -203,10 +221,12 @@ __global__ void __launch_bounds__(192, 1)
         const int kb1 = min(kb0 + p.kb_per_split, p.kb_total);
         for (int kb = kb0; kb < kb1 && pre < C::STAGES; ++kb, ++pre) {
           mbar_arrive_expect_tx(&full[pre], C::STAGE_BYTES);
+          int wx, wy;
+          weight_coords(p, kb, SWAP ? m_blk * C::BM : n_blk * BN, wx, wy);
           if (SWAP)
-            tma_load_2d(sA + pre * C::A_BYTES, &tmA, &full[pre], kb * C::BK, m_blk * C::BM);
+            tma_load_2d(sA + pre * C::A_BYTES, &tmA, &full[pre], wx, wy);
           else
-            tma_load_2d(sB + pre * C::B_BYTES, &tmB, &full[pre], kb * C::BK, n_blk * BN);
+            tma_load_2d(sB + pre * C::B_BYTES, &tmB, &full[pre], wx, wy);
         }
       }
       pdl_wait();
@@ -232,8 +252,15 @@ __global__ void __launch_bounds__(192, 1)
               break;
             }
             mbar_arrive_expect_tx(&full[stage], C::STAGE_BYTES);
-            tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
-            tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
+            int wx, wy;
+            weight_coords(p, kb, SWAP ? m_blk * C::BM : n_blk * BN, wx, wy);
+            if (SWAP) {
+              tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], wx, wy);
+              tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], kb * C::BK, n_blk * BN);
+            } else {
+              tma_load_2d(sA + stage * C::A_BYTES, &tmA, &full[stage], kb * C::BK, m_blk * C::BM);
+              tma_load_2d(sB + stage * C::B_BYTES, &tmB, &full[stage], wx, wy);
+            }
           }
           ++issued;
           if (++stage == C::STAGES) {

@@ -649,6 +649,39 @@ cudaError_t launch_pack_gate_up(const bf16* gate, const bf16* up, int F, int Fp,
   return cudaGetLastError();
 }
 
+// dst = src [N][K] (row pitch ld elements) in blocks of 256 rows x 64 columns: element (n, k) at
+// ((n / 256) * (Kp / 64) + k / 64) * 16384 + (n % 256) * 64 + k % 64 for n < ceil(N / 256) * 256
+// and k < Kp; rows >= N and columns >= K are zero.  One 16-byte chunk of dst per step, written in
+// order; vec: src and ld allow 16-byte loads.
+__global__ void block_rows_kernel(const bf16* src, int64_t N, int K, int64_t ld, int Kp, bool vec, bf16* dst) {
+  const int64_t kbs = Kp / 64;
+  const int64_t chunks = (N + 255) / 256 * 256 * (Kp / 8);
+  for (int64_t c = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; c < chunks; c += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t blk = c >> 11;  // 256 rows x 8 chunks per block
+    const int in = (int)(c & 2047);
+    const int64_t n = (blk / kbs) * 256 + (in >> 3);
+    const int k = (int)(blk % kbs) * 64 + (in & 7) * 8;
+    uint4 v = make_uint4(0, 0, 0, 0);
+    if (n < N) {
+      const bf16* row = src + n * ld;
+      if (vec && k + 8 <= K) {
+        v = *reinterpret_cast<const uint4*>(row + k);
+      } else {
+        alignas(16) unsigned short t[8];
+        for (int j = 0; j < 8; ++j) t[j] = k + j < K ? __bfloat16_as_ushort(row[k + j]) : (unsigned short)0;
+        v = *reinterpret_cast<const uint4*>(t);
+      }
+    }
+    reinterpret_cast<uint4*>(dst)[c] = v;
+  }
+}
+cudaError_t launch_block_rows(const bf16* src, int64_t N, int K, int64_t ld, int Kp, bf16* dst, cudaStream_t s) {
+  if (N < 1 || K < 1 || K > Kp || Kp % 64 || ld < K) return cudaErrorInvalidValue;
+  const bool vec = (reinterpret_cast<uintptr_t>(src) & 15) == 0 && ld % 8 == 0;
+  block_rows_kernel<<<2048, 256, 0, s>>>(src, N, K, ld, Kp, vec, dst);
+  return cudaGetLastError();
+}
+
 __global__ void bf16_to_f32_kernel(const bf16* src, int64_t n, float* dst) {
   for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x)
     dst[k] = __bfloat162float(src[k]);

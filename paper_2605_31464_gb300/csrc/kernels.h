@@ -57,12 +57,14 @@ int gemm_smem_bytes(int bn);
 // key of its largest element (see gemm_tc.cuh); the array must start at zero.
 // sample (device pointer, with argmax_keys): the keys rank the Gumbel-perturbed scores of token
 // t = *sample_step + sample_step_bias instead of the logits (temperature sampling, sampling.cuh).
+// w_blocked: the weight operand (A when swap, else B) is in the blocked layout of
+// launch_block_rows and its map has 64-element rows: {64, ceil(rows/256)*256 * K/64}, pitch 128 B.
 cudaError_t launch_gemm(const CUtensorMap& tmA, const CUtensorMap& tmB, int M, int N, int K, void* out,
                         int64_t ldo, int mode, int bn, int splits, int grid, int* err, cudaStream_t s,
                         int group_m = 0, bool swap = false, unsigned long long* argmax_keys = nullptr,
                         const SampleParams* sample = nullptr, const int32_t* sample_step = nullptr,
                         int sample_step_bias = 0, const RopeEpilogue* rope = nullptr,
-                        const NormFold* norm = nullptr);
+                        const NormFold* norm = nullptr, bool w_blocked = false);
 
 // ------------------------------------------------------------------ attention
 struct PrefillAttnArgs {
@@ -182,6 +184,10 @@ cudaError_t launch_build_prompts(const int32_t* inc_ids, const int32_t* inc_off,
                                  const int32_t* cand_off, const int32_t* prompt_off, int B, int T, int32_t* out,
                                  cudaStream_t s, int shared_inc = -1);
 cudaError_t launch_pack_gate_up(const bf16* gate, const bf16* up, int F, int Fp, int d, bf16* dst, cudaStream_t s);
+// Weight layout of the GEMMs (w_blocked): dst = src [N][K] (row pitch ld elements) in blocks of
+// 256 rows x 64 columns, [ceil(N/256)][Kp/64][256][64], zero beyond row N and column K
+// (Kp a multiple of 64, K <= Kp).  dst holds ceil(N/256) * 256 * Kp elements.
+cudaError_t launch_block_rows(const bf16* src, int64_t N, int K, int64_t ld, int Kp, bf16* dst, cudaStream_t s);
 cudaError_t launch_bf16_to_f32(const bf16* src, int64_t n, float* dst, cudaStream_t s);
 cudaError_t launch_rope_table(float theta, int hd, int max_seq, float2* cs, cudaStream_t s);
 cudaError_t launch_read_kv(const bf16* k_cache, const bf16* v_cache, const int32_t* block_table, int max_pages,

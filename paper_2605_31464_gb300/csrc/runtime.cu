@@ -321,7 +321,13 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
   *splits = std::max(1, s);
 }
 
+// Rows of a stored weight matrix: the GEMMs read every weight matrix in blocks of 256 rows x 64
+// columns (launch_block_rows), so N is rounded up to whole blocks of zero rows.
+int64_t weight_rows(int64_t n) { return (n + 255) / 256 * 256; }
+
 // n_alg / k_alg: the unpadded output width and contraction length (algorithmic work).
+// W is a weight matrix of the model, stored blocked (see weight_rows).
+
 // keys: ask the LM-head GEMM to fuse the greedy arg max (*fused tells whether it could).
 int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* out, int64_t ldo, int mode,
          cudaStream_t s, bool decode, int64_t n_alg = 0, int64_t k_alg = 0, unsigned long long* keys = nullptr,
@@ -338,12 +344,13 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
     splits = 1;
   }
   CUtensorMap ta, tb;
+  const uint64_t w_rows64 = (uint64_t)weight_rows(N) * (uint64_t)(K / 64);  // 64-element rows of W
   if (swap) {
-    TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, 128, &ta));
+    TRY(get_map(m, W, 64, w_rows64, 128, &ta));
     TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, (uint32_t)bn, &tb));
   } else {
     TRY(get_map(m, A, (uint64_t)K, (uint64_t)M, 128, &ta));
-    TRY(get_map(m, W, (uint64_t)K, (uint64_t)N, (uint32_t)bn, &tb));
+    TRY(get_map(m, W, 64, w_rows64, (uint32_t)bn, &tb));
   }
   const double na = n_alg ? n_alg : N, ka = k_alg ? k_alg : K;
   const double out_bytes =
@@ -354,10 +361,10 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
   if (fused) *fused = use_keys;
   if (swap)
     CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, true,
-                       use_keys ? keys : nullptr, sample, sample_step, sample_bias));
+                       use_keys ? keys : nullptr, sample, sample_step, sample_bias, nullptr, nullptr, true));
   else
     CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, m->sms, m->err, s, 0, false, nullptr, nullptr,
-                       nullptr, 0, rope, norm));
+                       nullptr, 0, rope, norm, true));
   m->launches += 1;
   return GF_OK;
 }
@@ -1065,15 +1072,15 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   m->layers.resize(m->L);
   for (int l = 0; l < m->L && rc == GF_OK; ++l) {
     gf_model::Layer& W = m->layers[l];
-    rc = dalloc(m, &W.qkv, (size_t)m->qkv_dim * d);
-    if (!rc) rc = dalloc(m, &W.o, (size_t)d * m->q_dim);
-    if (!rc) rc = dalloc(m, &W.gu, (size_t)2 * m->ffn_pad * d);
-    if (!rc) rc = dalloc(m, &W.down, (size_t)d * m->ffn_pad);
+    rc = dalloc(m, &W.qkv, (size_t)weight_rows(m->qkv_dim) * d);
+    if (!rc) rc = dalloc(m, &W.o, (size_t)weight_rows(d) * m->q_dim);
+    if (!rc) rc = dalloc(m, &W.gu, (size_t)weight_rows(2 * m->ffn_pad) * d);
+    if (!rc) rc = dalloc(m, &W.down, (size_t)weight_rows(d) * m->ffn_pad);
     if (!rc) rc = dalloc(m, &W.attn_norm, d);
     if (!rc) rc = dalloc(m, &W.ffn_norm, d);
   }
   if (!rc) rc = dalloc(m, &m->embed, (size_t)m->vocab * d);
-  if (!rc) rc = dalloc(m, &m->head, (size_t)m->vocab * d);
+  if (!rc) rc = dalloc(m, &m->head, (size_t)weight_rows(m->vocab) * d);
   if (!rc) rc = dalloc(m, &m->final_norm, d);
   // ---- KV pool, tables
   const size_t cache_elems = (size_t)m->L * m->num_pages * m->nkv * 64 * hd;
@@ -1119,35 +1126,50 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (!rc) rc = dalloc(m, &m->samp, 1);
   if (rc) return bail(rc);
 
-  // ---- pack weights
+  // ---- pack weights: q, k, v rows stacked and gate/up interleaved (row-major, in a scratch
+  // buffer), then every GEMM weight stored in 256 x 64 blocks
   auto cp = [&](void* dst, const void* src, size_t bytes) {
     return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyDeviceToDevice, s);
   };
+  struct Scratch {
+    bf16* p = nullptr;
+    ~Scratch() {
+      if (p) cudaFree(p);
+    }
+  } tmp;
+  if (cudaMalloc(&tmp.p, std::max((size_t)m->qkv_dim, (size_t)2 * m->ffn_pad) * d * sizeof(bf16)) != cudaSuccess) {
+    cudaGetLastError();
+    return bail(fail(GF_ENOMEM, "weight packing scratch"));
+  }
   cudaError_t e = cudaSuccess;
   const size_t qb = (size_t)m->q_dim * d * 2, kb = (size_t)m->nkv * hd * d * 2;
   for (int l = 0; l < m->L && e == cudaSuccess; ++l) {
     gf_model::Layer& W = m->layers[l];
     if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->w_gate[l] || !w->w_up[l] || !w->w_down[l] ||
-        !w->attn_norm[l] || !w->ffn_norm[l])
+        !w->attn_norm[l] || !w->ffn_norm[l]) {
+      cudaStreamSynchronize(s);
       return bail(fail(GF_EINVAL, "null weight pointer in layer %d", l));
-    e = cp(W.qkv, w->wq[l], qb);
-    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(W.qkv) + qb, w->wk[l], kb);
-    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(W.qkv) + qb + kb, w->wv[l], kb);
-    if (e == cudaSuccess) e = cp(W.o, w->wo[l], (size_t)d * m->q_dim * 2);
+    }
+    e = cp(tmp.p, w->wq[l], qb);
+    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(tmp.p) + qb, w->wk[l], kb);
+    if (e == cudaSuccess) e = cp(reinterpret_cast<char*>(tmp.p) + qb + kb, w->wv[l], kb);
+    if (e == cudaSuccess) e = gf::launch_block_rows(tmp.p, m->qkv_dim, d, d, d, W.qkv, s);
+    if (e == cudaSuccess)
+      e = gf::launch_block_rows(reinterpret_cast<const bf16*>(w->wo[l]), d, m->q_dim, m->q_dim, m->q_dim, W.o, s);
     if (e == cudaSuccess)
       e = gf::launch_pack_gate_up(reinterpret_cast<const bf16*>(w->w_gate[l]),
-                                  reinterpret_cast<const bf16*>(w->w_up[l]), m->ffn, m->ffn_pad, d, W.gu, s);
-    if (e == cudaSuccess) e = cudaMemsetAsync(W.down, 0, (size_t)d * m->ffn_pad * 2, s);
+                                  reinterpret_cast<const bf16*>(w->w_up[l]), m->ffn, m->ffn_pad, d, tmp.p, s);
+    if (e == cudaSuccess) e = gf::launch_block_rows(tmp.p, 2 * m->ffn_pad, d, d, d, W.gu, s);
     if (e == cudaSuccess)
-      e = cudaMemcpy2DAsync(W.down, (size_t)m->ffn_pad * 2, w->w_down[l], (size_t)m->ffn * 2, (size_t)m->ffn * 2, d,
-                            cudaMemcpyDeviceToDevice, s);
+      e = gf::launch_block_rows(reinterpret_cast<const bf16*>(w->w_down[l]), d, m->ffn, m->ffn, m->ffn_pad, W.down,
+                                s);
     if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->attn_norm[l]), d, W.attn_norm, s);
     if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->ffn_norm[l]), d, W.ffn_norm, s);
   }
   m->weight_bytes = (double)m->L * ((double)m->qkv_dim * d + (double)d * m->q_dim + 2.0 * m->ffn * d +
                                     (double)d * m->ffn) * 2 + (double)m->vocab * d * 2;
   if (e == cudaSuccess) e = cp(m->embed, w->embed, (size_t)m->vocab * d * 2);
-  if (e == cudaSuccess) e = cp(m->head, w->lm_head, (size_t)m->vocab * d * 2);
+  if (e == cudaSuccess) e = gf::launch_block_rows(reinterpret_cast<const bf16*>(w->lm_head), m->vocab, d, d, d, m->head, s);
   if (e == cudaSuccess) e = gf::launch_bf16_to_f32(reinterpret_cast<const bf16*>(w->final_norm), d, m->final_norm, s);
   if (e == cudaSuccess) e = gf::launch_rope_table(c.rope_theta, hd, c.max_seq, m->rope_cs, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(m->dqkv, 0, Bm * m->qkv_dim * sizeof(float), s);
@@ -1155,7 +1177,10 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   if (e == cudaSuccess) e = cudaMemsetAsync(m->seq_len, 0, Bm * sizeof(int32_t), s);
   if (e == cudaSuccess) e = cudaMemsetAsync(m->keys, 0, Bm * sizeof(unsigned long long), s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
-  if (e != cudaSuccess) return bail(fail(GF_ECUDA, "weight packing failed: %s", cudaGetErrorString(e)));
+  if (e != cudaSuccess) {
+    cudaStreamSynchronize(s);  // nothing may still read the scratch buffer when it is freed
+    return bail(fail(GF_ECUDA, "weight packing failed: %s", cudaGetErrorString(e)));
+  }
 
   // ---- host state
   m->h_bt.assign((size_t)m->B_max * m->max_pages, -1);
