@@ -250,6 +250,26 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
  * launch gave up waiting. */
 int gf_gemm_status(void* stream);
 
+/* ---- planning queries (host arithmetic only: no device work, no GPU needed) --
+ * gf_plan_gemm: the tiling the model's GEMMs, and gf_gemm_bf16 with
+ * bn = splits = 0, use for an M x N x K product in `mode` (GF_GEMM_*) on a GPU
+ * with `sms` SMs.
+ *   *swap    1: the weights are the 128-row MMA operand and the M activation
+ *            rows the narrow one (decode; M <= 128).  0: M rows in 128-row tiles.
+ *   *bn      tile width: activation rows per tile when swapped (32, 64 or 128),
+ *            else output columns per tile (64, 128 or 256).
+ *   *splits  split-K factor (> 1 only in GF_GEMM_ATOMIC_F32 mode).
+ * Returns GF_OK, or GF_EINVAL for sms, M, N or K < 1, a bad mode or a null
+ * output pointer.  (Inside the model a GEMM whose epilogue applies a folded
+ * RMSNorm is never swapped.) */
+int gf_plan_gemm(int32_t sms, int32_t M, int32_t N, int32_t K, int32_t mode, int32_t* bn, int32_t* splits,
+                 int32_t* swap);
+/* gf_plan_decode_chunk: keys per decode-attention CTA (1024, 512 or 256) for
+ * B sequences of up to max_ctx cached tokens and n_kv KV heads: the longest
+ * chunk that still gives every SM two CTAs.  Returns the chunk, or GF_EINVAL
+ * for a size < 1. */
+int32_t gf_plan_decode_chunk(int32_t B, int32_t n_kv, int32_t max_ctx, int32_t sms);
+
 /* Decode attention over a paged KV cache, the step a decode token spends on
  * its context (one query token per sequence, grouped-query heads):
  *   out[b, h, :] = sum_j softmax_j(q[b,h,:] . k_j / sqrt(hd)) v_j  over the

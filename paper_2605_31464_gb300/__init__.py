@@ -47,7 +47,7 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
            "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select",
-           "gf_forecast_batch_sampled", "gf_sample_tokens"]
+           "gf_forecast_batch_sampled", "gf_sample_tokens", "gf_plan_gemm", "gf_plan_decode_chunk"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
 GF_PROF_PREFILL_GEMM, GF_PROF_DECODE_GEMM, GF_PROF_PREFILL_ATTN, GF_PROF_DECODE_ATTN, GF_PROF_DECODE_STEPS = range(5)
@@ -90,6 +90,9 @@ def load(path: str = LIB_PATH):
         "gf_gemm_bf16": ([_p, _p, _c_i32, _c_i32, _c_i32, _p, _c_i64, _c_i32, _c_i32, _c_i32, _c_i32, _p],
                          ctypes.c_int),
         "gf_gemm_status": ([_p], ctypes.c_int),
+        "gf_plan_gemm": ([_c_i32, _c_i32, _c_i32, _c_i32, _c_i32, ctypes.POINTER(_c_i32), ctypes.POINTER(_c_i32),
+                          ctypes.POINTER(_c_i32)], ctypes.c_int),
+        "gf_plan_decode_chunk": ([_c_i32, _c_i32, _c_i32, _c_i32], _c_i32),
         "gf_decode_attention_workspace": ([_c_i32, _c_i32, _c_i32, _c_i32], ctypes.c_size_t),
         "gf_decode_attention_static": ([_p, _p, _p, _c_i64, _p, _c_i32, _p, _c_i32, _c_i32, _c_i32, _c_i32, _c_i32,
                                         _p, _p], ctypes.c_int),
@@ -235,6 +238,21 @@ def gf_gemm_bf16(A, W, M, N, K, out, ldo, mode, bn, splits, group_m, stream):
 
 def gf_gemm_status(stream):
     _check(load().gf_gemm_status(stream))
+
+
+def gf_plan_gemm(sms, M, N, K, mode) -> dict:
+    """The GEMM tiling the library chooses (host arithmetic only; needs no GPU)."""
+    bn, splits, swap = _c_i32(), _c_i32(), _c_i32()
+    _check(load().gf_plan_gemm(sms, M, N, K, mode, ctypes.byref(bn), ctypes.byref(splits), ctypes.byref(swap)))
+    return dict(bn=bn.value, splits=splits.value, swap=bool(swap.value))
+
+
+def gf_plan_decode_chunk(B, n_kv, max_ctx, sms) -> int:
+    """Keys per decode-attention CTA (host arithmetic only; needs no GPU)."""
+    rc = int(load().gf_plan_decode_chunk(B, n_kv, max_ctx, sms))
+    if rc not in (256, 512, 1024):
+        raise GfError(rc, load().gf_last_error().decode())
+    return rc
 
 
 def gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx) -> int:

@@ -1462,6 +1462,30 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   return GF_OK;
 }
 
+static_assert(GF_GEMM_STORE_F32 == gf::kStoreF32 && GF_GEMM_ADD_F32 == gf::kAddF32 &&
+                  GF_GEMM_ATOMIC_F32 == gf::kAtomicF32 && GF_GEMM_STORE_BF16 == gf::kStoreBF16 &&
+                  GF_GEMM_SWIGLU == gf::kSwiGLU,
+              "public GEMM modes are the kernel's modes");
+
+int gf_plan_gemm(int32_t sms, int32_t M, int32_t N, int32_t K, int32_t mode, int32_t* bn, int32_t* splits,
+                 int32_t* swap) {
+  if (!bn || !splits || !swap) return fail(GF_EINVAL, "null output pointer");
+  if (sms < 1 || M < 1 || N < 1 || K < 1) return fail(GF_EINVAL, "sizes must be positive");
+  if (mode < GF_GEMM_STORE_F32 || mode > GF_GEMM_SWIGLU) return fail(GF_EINVAL, "bad GEMM mode");
+  int b = 0, sp = 1;
+  bool sw = false;
+  plan_gemm(sms, M, N, K, mode, &b, &sp, &sw);
+  *bn = b;
+  *splits = sp;
+  *swap = sw ? 1 : 0;
+  return GF_OK;
+}
+
+int32_t gf_plan_decode_chunk(int32_t B, int32_t n_kv, int32_t max_ctx, int32_t sms) {
+  if (B < 1 || n_kv < 1 || max_ctx < 1 || sms < 1) return fail(GF_EINVAL, "sizes must be positive");
+  return decode_chunk(B, n_kv, max_ctx, sms);
+}
+
 int gf_gemm_status(void* stream) {
   CU(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
   if (!g_gemm_err) return GF_OK;  // shared by gf_gemm_bf16 and gf_decode_attention
