@@ -14,6 +14,7 @@
 #include "gf.h"
 #include "gemm_tc.cuh"
 #include "kernels.h"
+#include "page_pool.h"
 
 using gf::bf16;
 
@@ -183,11 +184,12 @@ struct gf_model {
   float* out_small = nullptr;  // host-variant outputs on the device
   int* err = nullptr;
 
-  // host mirrors
-  std::vector<int32_t> h_bt, h_len;
+  // host state: block tables and the reference-counted page pool; per slot its length and
+  // whether it is live; the free slots
+  gf::KvPagePool pool;
+  std::vector<int32_t> h_len;
   std::vector<char> live;
-  std::vector<int32_t> free_pages, free_slots;
-  std::vector<int32_t> page_ref;  // block-table entries that point at each page (shared prefixes)
+  std::vector<int32_t> free_slots;
   std::vector<Capture> caps;
   std::map<std::tuple<const void*, uint64_t, uint64_t, uint32_t>, CUtensorMap> maps;
   Staging staging;
@@ -399,47 +401,21 @@ int fire_captures(gf_model* m, int layer, const float* base, const int32_t* offs
   return GF_OK;
 }
 
-int alloc_pages(gf_model* m, int slot, int first, int count, std::vector<std::pair<int, int>>* undo) {
-  for (int j = first; j < first + count; ++j) {
-    if (m->h_bt[(int64_t)slot * m->max_pages + j] >= 0) continue;
-    if (m->free_pages.empty()) return fail(GF_ECAPACITY, "KV page pool exhausted");
-    const int p = m->free_pages.back();
-    m->free_pages.pop_back();
-    m->h_bt[(int64_t)slot * m->max_pages + j] = p;
-    m->page_ref[p] = 1;
-    undo->push_back({slot, j});
-  }
+int alloc_pages(gf_model* m, int slot, int first, int count, gf::KvPagePool::Undo* undo) {
+  if (!m->pool.alloc(slot, first, count, undo)) return fail(GF_ECAPACITY, "KV page pool exhausted");
   return GF_OK;
 }
 
-// Point entries [0, count) of `slot` at the pages of `from` (copy-free sharing of a cached prefix).
-void share_pages(gf_model* m, int slot, int from, int count, std::vector<std::pair<int, int>>* undo) {
-  for (int j = 0; j < count; ++j) {
-    const int p = m->h_bt[(int64_t)from * m->max_pages + j];
-    m->h_bt[(int64_t)slot * m->max_pages + j] = p;
-    m->page_ref[p] += 1;
-    undo->push_back({slot, j});
-  }
-}
-
-void drop_page(gf_model* m, int32_t& e) {
-  if (e >= 0 && --m->page_ref[e] == 0) m->free_pages.push_back(e);
-  e = -1;
-}
-
-void undo_pages(gf_model* m, const std::vector<std::pair<int, int>>& undo) {
-  for (auto it = undo.rbegin(); it != undo.rend(); ++it) drop_page(m, m->h_bt[(int64_t)it->first * m->max_pages + it->second]);
-}
-
 void release_slot(gf_model* m, int slot) {
-  for (int j = 0; j < m->max_pages; ++j) drop_page(m, m->h_bt[(int64_t)slot * m->max_pages + j]);
+  m->pool.clear(slot);
   m->h_len[slot] = 0;
   m->live[slot] = 0;
   m->free_slots.push_back(slot);
 }
 
 int upload_block_table(gf_model* m, cudaStream_t s) {
-  return upload(m->staging, m->bt, m->h_bt.data(), m->h_bt.size() * sizeof(int32_t), s);
+  const std::vector<int32_t>& t = m->pool.table();
+  return upload(m->staging, m->bt, t.data(), t.size() * sizeof(int32_t), s);
 }
 
 // Prefill of B packed prompts already on the device.  `reserve` extra
@@ -466,7 +442,7 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   if ((int)m->free_slots.size() < B) return fail(GF_ECAPACITY, "no free sequence slots");
   // slots and pages
   std::vector<int32_t> slots(B);
-  std::vector<std::pair<int, int>> undo;
+  gf::KvPagePool::Undo undo;
   for (int b = 0; b < B; ++b) {
     slots[b] = m->free_slots.back();
     m->free_slots.pop_back();
@@ -474,10 +450,10 @@ int prefill_impl(gf_model* m, int B, const int32_t* ids, const int32_t* offsets,
   const int shared = past / 64;
   for (int b = 0; b < B; ++b) {
     const int len = offsets[b + 1] - offsets[b];
-    if (shared > 0) share_pages(m, slots[b], share_slot, shared, &undo);
+    if (shared > 0) m->pool.share(slots[b], share_slot, shared, &undo);
     const int rc = alloc_pages(m, slots[b], shared, (past + len + reserve + 63) / 64 - shared, &undo);
     if (rc != GF_OK) {
-      undo_pages(m, undo);
+      m->pool.rollback(undo);
       for (int bb = B - 1; bb >= 0; --bb) m->free_slots.push_back(slots[bb]);
       return rc;
     }
@@ -806,12 +782,12 @@ int prepare_decode(gf_model* m, int B, const int32_t* h, cudaStream_t s) {
     seen[h[b]] = 1;
     if (m->h_len[h[b]] + 1 > m->cfg.max_seq) return fail(GF_ECAPACITY, "sequence %d reached max_seq", h[b]);
   }
-  std::vector<std::pair<int, int>> undo;
+  gf::KvPagePool::Undo undo;
   for (int b = 0; b < B; ++b) {
     const int pos = m->h_len[h[b]];
     const int rc = alloc_pages(m, h[b], pos / 64, 1, &undo);
     if (rc != GF_OK) {
-      undo_pages(m, undo);
+      m->pool.rollback(undo);
       return rc;
     }
   }
@@ -858,7 +834,7 @@ int assemble_prompts(gf_model* m, int B, const int32_t* inc_ids, const int32_t* 
 // rows and h is released.
 int fork_sequences(gf_model* m, int B, int R, const int32_t* h, int n_decode, std::vector<int32_t>& rows,
                    std::vector<int32_t>& jobs) {
-  std::vector<std::pair<int, int>> unused;
+  gf::KvPagePool::Undo unused;
   for (int b = 0; b < B; ++b) rows[(size_t)b * R] = h[b];
   int rc = GF_OK;
   for (int b = 0; b < B && rc == GF_OK; ++b) {
@@ -873,11 +849,11 @@ int fork_sequences(gf_model* m, int B, int R, const int32_t* h, int n_decode, st
       m->live[slot] = 1;
       m->h_len[slot] = len;
       rows[(size_t)b * R + j] = slot;
-      share_pages(m, slot, h[b], full, &unused);
+      m->pool.share(slot, h[b], full, &unused);
       rc = alloc_pages(m, slot, full, (len + n_decode + 63) / 64 - full, &unused);
       const bool partial = len % 64 != 0;
-      jobs.insert(jobs.end(), {h[b], slot, partial ? m->h_bt[(int64_t)h[b] * m->max_pages + full] : -1,
-                               partial ? m->h_bt[(int64_t)slot * m->max_pages + full] : -1});
+      jobs.insert(jobs.end(), {h[b], slot, partial ? m->pool.entry(h[b], full) : -1,
+                               partial ? m->pool.entry(slot, full) : -1});
     }
   }
   if (rc != GF_OK) {
@@ -1008,7 +984,7 @@ const char* gf_last_error(void) { return g_err.c_str(); }
 
 int64_t gf_launch_count(const gf_model* m) { return m ? m->launches : 0; }
 
-int64_t gf_free_pages(const gf_model* m) { return m ? (int64_t)m->free_pages.size() : 0; }
+int64_t gf_free_pages(const gf_model* m) { return m ? m->pool.free_pages() : 0; }
 
 void gf_destroy(gf_model* m) {
   if (!m) return;
@@ -1183,12 +1159,9 @@ int gf_create(const gf_config* cfg, const gf_weights* w, void* stream, gf_model*
   }
 
   // ---- host state
-  m->h_bt.assign((size_t)m->B_max * m->max_pages, -1);
+  m->pool.init(m->B_max, m->max_pages, m->num_pages);
   m->h_len.assign(m->B_max, 0);
   m->live.assign(m->B_max, 0);
-  m->free_pages.reserve(m->num_pages);
-  m->page_ref.assign(m->num_pages, 0);
-  for (int64_t p = m->num_pages - 1; p >= 0; --p) m->free_pages.push_back((int32_t)p);
   for (int sl = m->B_max - 1; sl >= 0; --sl) m->free_slots.push_back(sl);
   const uint64_t rows = (uint64_t)m->L * m->num_pages * m->nkv * 64;
   if ((rc = make_map(&m->tm_k, m->k_cache, hd, rows, hd * 2, 64, 64))) return bail(rc);
