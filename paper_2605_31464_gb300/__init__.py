@@ -173,6 +173,7 @@ def gf_sample_tokens(B, logits, ld, V, seed, token_index, temperature, out_ids, 
 def sample_tokens(logits, seed, token_index, temperature, stream=None):
     """Temperature draw (Gumbel-max, counter-based) for each row of a [B, V] float32 CUDA tensor."""
     import torch
+    _check_tensor(logits, "logits", dtype=torch.float32, rows_strided=True)
     s = stream if stream is not None else torch.cuda.current_stream()
     out = torch.empty(logits.shape[0], dtype=torch.int32, device=logits.device)
     gf_sample_tokens(logits.shape[0], logits.data_ptr(), logits.stride(0), logits.shape[1], int(seed),
@@ -187,6 +188,7 @@ def gf_select(B, p, m_bins, x_cut, tau_disc, s_hat, order, disc, disc_pred, stre
 def select(p, m_bins, x_cut, tau_disc, stream=None):
     """Expected speedup, ranking and discovery score of a [B, 8] CUDA tensor of bin probabilities."""
     import torch
+    _check_tensor(p, "p", (p.shape[0], 8), torch.float32)
     s = stream if stream is not None else torch.cuda.current_stream()
     B = p.shape[0]
     m = np.ascontiguousarray(np.asarray(m_bins, dtype=np.float32))
@@ -278,6 +280,11 @@ def decode_attention(q, k_cache, v_cache, block_table, ctx_len, max_ctx, n_q, n_
     s = stream if stream is not None else torch.cuda.current_stream()
     B = q.shape[0]
     hd = k_cache.shape[-1]
+    _check_tensor(q, "q", (B, n_q * hd), torch.bfloat16)
+    _check_tensor(k_cache, "k_cache", (k_cache.shape[0], n_kv, 64, hd), torch.bfloat16)
+    _check_tensor(v_cache, "v_cache", (k_cache.shape[0], n_kv, hd, 64), torch.bfloat16)
+    _check_tensor(block_table, "block_table", (B, block_table.shape[1]), torch.int32)
+    _check_ids(ctx_len, "ctx_len", B)
     ws_bytes = gf_decode_attention_workspace(B, n_kv, hd, max_ctx)
     ws = torch.empty(ws_bytes, dtype=torch.uint8, device=q.device)
     out = torch.empty_like(q)
@@ -303,6 +310,12 @@ def gemm(A, W, out, mode=GF_GEMM_STORE_F32, bn=0, splits=0, stream=None, group_m
     s = stream if stream is not None else torch.cuda.current_stream()
     M, K = A.shape
     N = W.shape[0]
+    _check_tensor(A, "A", (M, K), torch.bfloat16)
+    _check_tensor(W, "W", (N, K), torch.bfloat16)
+    bf16_out = mode in (GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU)
+    _check_tensor(out, "out", dtype=torch.bfloat16 if bf16_out else torch.float32, rows_strided=True)
+    if out.shape[0] < M or out.shape[1] < (N // 2 if mode == GF_GEMM_SWIGLU else N):
+        raise ValueError(f"out: shape {tuple(out.shape)} too small for {M} x {N}")
     gf_gemm_bf16(A.data_ptr(), W.data_ptr(), M, N, K, out.data_ptr(), out.stride(0), mode, bn, splits, group_m,
                  s.cuda_stream)
 
@@ -317,6 +330,48 @@ def _ptr(a: np.ndarray):
     return a.ctypes.data_as(_p)
 
 
+def _check_tensor(t, name, shape=None, dtype=None, rows_strided=False):
+    """Refuse what the C ABI cannot see through a pointer: a wrong shape or dtype, a tensor
+    in host memory, or a layout other than row-major (rows_strided: any row stride)."""
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name}: expected a torch tensor, got {type(t).__name__}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected {tuple(shape)}")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    dense = (t.dim() == 2 and t.stride(1) == 1 and t.stride(0) >= t.shape[1]) if rows_strided else t.is_contiguous()
+    if not dense:
+        raise ValueError(f"{name}: layout not supported (strides {tuple(t.stride())})")
+    if not t.is_cuda:
+        raise ValueError(f"{name}: must be a CUDA tensor")
+
+
+def _check_ids(t, name, n):
+    """A 1-D int32 CUDA tensor holding at least the n ids the call reads."""
+    import torch
+    _check_tensor(t, name, dtype=torch.int32)
+    if t.dim() != 1 or t.numel() < n:
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected 1-D with at least {n} ids")
+
+
+def _check_weights(shape, weights: dict):
+    """Shapes and dtypes gf_create reads (it copies bytes by those shapes)."""
+    import torch
+    d, hd, L = shape.d_model, shape.head_dim, shape.layers
+    bf16 = torch.bfloat16
+    for name, shp in (("embed", (shape.vocab, d)), ("lm_head", (shape.vocab, d)), ("final_norm", (d,))):
+        _check_tensor(weights[name], name, shp, bf16)
+    per_layer = {"attn_norm": (d,), "ffn_norm": (d,), "wq": (shape.n_q * hd, d), "wk": (shape.n_kv * hd, d),
+                 "wv": (shape.n_kv * hd, d), "wo": (d, shape.n_q * hd), "w_gate": (shape.ffn, d),
+                 "w_up": (shape.ffn, d), "w_down": (d, shape.ffn)}
+    for name, shp in per_layer.items():
+        if len(weights[name]) != L:
+            raise ValueError(f"{name}: {len(weights[name])} tensors for {L} layers")
+        for l, t in enumerate(weights[name]):
+            _check_tensor(t, f"{name}[{l}]", shp, bf16)
+
+
 class Model:
     """A model on the current CUDA device.
 
@@ -329,6 +384,7 @@ class Model:
     def __init__(self, shape, weights: dict, max_batch: int, max_seq: int, max_prefill_tokens: int,
                  kv_pages: int = 0, stream=None):
         import torch
+        _check_weights(shape, weights)
         self.torch = torch
         self.shape = shape
         self.stream = stream if stream is not None else torch.cuda.current_stream()
@@ -372,6 +428,7 @@ class Model:
         torch = self.torch
         off = _i32_host(offsets)
         B = len(off) - 1
+        _check_ids(ids, "ids", int(off[-1]))
         handles = np.zeros(B, dtype=np.int32)
         logits = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
         nxt = torch.empty(B, dtype=torch.int32, device="cuda")
@@ -383,6 +440,7 @@ class Model:
         torch = self.torch
         h = _i32_host(handles)
         B = len(h)
+        _check_ids(ids, "ids", B)
         logits = torch.empty(B, self.shape.vocab, dtype=torch.float32, device="cuda") if want_logits else None
         nxt = torch.empty(B, dtype=torch.int32, device="cuda")
         gf_decode_step(self.handle, B, _ptr(h), ids.data_ptr(), logits.data_ptr() if logits is not None else None,
@@ -398,6 +456,8 @@ class Model:
         torch = self.torch
         io, co, vid = _i32_host(inc_offsets), _i32_host(cand_offsets), _i32_host(verdict_ids)
         B, K = len(io) - 1, len(vid)
+        _check_ids(inc_ids, "inc_ids", int(io[-1]))
+        _check_ids(cand_ids, "cand_ids", int(co[-1]))
         p = torch.empty(B, K, dtype=torch.float32, device="cuda")
         conf = torch.empty(B, dtype=torch.float32, device="cuda")
         arg = torch.empty(B, dtype=torch.int32, device="cuda")
@@ -416,6 +476,8 @@ class Model:
         torch = self.torch
         co, vid = _i32_host(cand_offsets), _i32_host(verdict_ids)
         B, K = len(co) - 1, len(vid)
+        _check_ids(prefix_ids, "prefix_ids", prefix_ids.numel())
+        _check_ids(cand_ids, "cand_ids", int(co[-1]))
         p = torch.empty(B, K, dtype=torch.float32, device="cuda")
         conf = torch.empty(B, dtype=torch.float32, device="cuda")
         arg = torch.empty(B, dtype=torch.int32, device="cuda")
@@ -436,6 +498,8 @@ class Model:
         torch = self.torch
         io, co, vid = _i32_host(inc_offsets), _i32_host(cand_offsets), _i32_host(verdict_ids)
         B, K = len(io) - 1, len(vid)
+        _check_ids(inc_ids, "inc_ids", int(io[-1]))
+        _check_ids(cand_ids, "cand_ids", int(co[-1]))
         BR = B * repeats
         f32 = dict(dtype=torch.float32, device="cuda")
         p, conf = torch.empty(BR, K, **f32), torch.empty(BR, **f32)
@@ -503,6 +567,7 @@ def verdict(logits, verdict_ids, tau, stream=None):
     import torch
     s = stream if stream is not None else torch.cuda.current_stream()
     vid = _i32_host(verdict_ids)
+    _check_tensor(logits, "logits", dtype=torch.float32, rows_strided=True)
     B, K = logits.shape[0], len(vid)
     p = torch.empty(B, K, dtype=torch.float32, device=logits.device)
     conf = torch.empty(B, dtype=torch.float32, device=logits.device)
