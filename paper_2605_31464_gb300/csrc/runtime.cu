@@ -287,7 +287,7 @@ void plan_gemm(int sms, int M, int N, int K, int mode, int* bn, int* splits, boo
   const int num_m = (M + 127) / 128;
   *splits = 1;
   *swap = false;
-  // SwiGLU above 64 rows: row-major 256-wide weight tiles move fewer activation bytes per weight byte
+  // SwiGLU above 64 rows: non-swapped 256-wide weight tiles move fewer activation bytes per weight byte
   // than 128-wide swapped ones (measured about 10 % faster at 96-128 rows)
   const bool swap_ok = mode == gf::kStoreF32 || mode == gf::kAtomicF32 || (mode == gf::kSwiGLU && M <= 64);
   if (M <= 128 && N % 32 == 0 && swap_ok) {
@@ -340,7 +340,7 @@ int gemm(gf_model* m, const bf16* A, int M, int K, const bf16* W, int N, void* o
   bool swap;
   plan_gemm(m->sms, M, N, K, mode, &bn, &splits, &swap);
   if (norm && swap) {
-    // the folded RMSNorm is applied by the row-major (non-swapped) epilogues only
+    // the folded RMSNorm is applied by the non-swapped epilogues only
     swap = false;
     bn = 128;
     splits = 1;
@@ -1419,7 +1419,7 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   bool swap = false;
   plan_gemm(sms, M, N, K, mode, &pbn, &psplits, &swap);
   const bool bn_given = bn != 0;
-  if (bn_given) swap = false;  // an explicit tile width asks for the row-major tiling
+  if (bn_given) swap = false;  // an explicit tile width asks for the non-swapped tiling
   if (!bn_given) bn = pbn;
   if (splits <= 0) splits = bn_given ? 1 : psplits;
   CUtensorMap ta, tb;

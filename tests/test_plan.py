@@ -5,7 +5,7 @@ The planner's choices must always satisfy what the GEMM kernel can run (a
 swapped tile holds every activation row, split-K only with atomic
 accumulation, each split at least four 64-column k-blocks), and they must
 follow the stated rules: swap operands for decode-sized M, 256-wide tiles once
-there are four 128-row blocks, SwiGLU above 64 rows on row-major tiles, and
+there are four 128-row blocks, SwiGLU above 64 rows on non-swapped tiles, and
 about one wave of (tile, split) units for split-K.
 """
 import itertools
@@ -86,7 +86,7 @@ def test_decode_shapes_of_the_7b_model():
     assert plan(32, 37888, 3584, gf.GF_GEMM_SWIGLU) == dict(bn=32, splits=1, swap=True)
     assert plan(32, 3584, 18944, gf.GF_GEMM_ATOMIC_F32) == dict(bn=32, splits=5, swap=True)
     assert plan(32, 152064, 3584, gf.GF_GEMM_STORE_F32) == dict(bn=32, splits=1, swap=True)
-    # 128 sequences: SwiGLU moves to row-major 256-wide tiles
+    # 128 sequences: SwiGLU moves to non-swapped 256-wide tiles
     assert plan(128, 37888, 3584, gf.GF_GEMM_SWIGLU) == dict(bn=256, splits=1, swap=False)
     assert plan(128, 4608, 3584, gf.GF_GEMM_ATOMIC_F32)["swap"]
 
