@@ -55,8 +55,8 @@ typedef struct gf_config {
   int32_t n_q;         /* query heads */
   int32_t n_kv;        /* key/value heads; n_q % n_kv == 0, n_q / n_kv <= 16 */
   int32_t head_dim;    /* 64 or 128 */
-  int32_t ffn;         /* SwiGLU width */
-  int32_t vocab;
+  int32_t ffn;         /* SwiGLU width (padded to a multiple of 64 inside, with zero weights) */
+  int32_t vocab;       /* multiple of 32, >= 32 */
   float rope_theta;
   float rms_eps;
   int32_t max_batch;   /* sequence slots (concurrent sequences), <= 1024 */
