@@ -53,7 +53,7 @@ def _decode_attn(a):
     rng = np.random.default_rng(0)
     table = torch.from_numpy(rng.permutation(n_pages).astype(np.int32).reshape(a.B, pages_per)).cuda()
     kc = torch.randn(n_pages, a.n_kv, 64, hd, device="cuda").bfloat16()
-    vc = torch.randn(n_pages, a.n_kv, 64, hd, device="cuda").bfloat16()
+    vc = torch.randn(n_pages, a.n_kv, hd, 64, device="cuda").bfloat16()  # pages stored transposed
     q = torch.randn(a.B, a.n_q * hd, device="cuda").bfloat16()
     ctx = torch.full((a.B,), a.ctx, dtype=torch.int32, device="cuda")
     s = torch.cuda.current_stream()
