@@ -94,3 +94,48 @@ def test_sampling_argument_validation_needs_no_gpu(lib):
                                      vid.ctypes.data_as(ctypes.c_void_p), 2, 0.8, dummy, dummy, dummy, dummy, None,
                                      None, None, None, None, None, None)
     assert e.value.code == gf.GF_EINVAL
+
+
+def test_decode_attention_argument_validation_needs_no_gpu(lib):
+    d = ctypes.c_void_p(256)
+    ws = gf.gf_decode_attention_workspace(4, 2, 128, 1000)
+    ok = dict(q=d, k=d, v=d, num_pages=64, table=d, max_pages=16, ctx=d, max_ctx=1000, B=4, n_q=8, n_kv=2, hd=128,
+              out=d, ws=d, ws_bytes=ws)
+
+    def call(**kw):
+        a = dict(ok, **kw)
+        return (a["q"], a["k"], a["v"], a["num_pages"], a["table"], a["max_pages"], a["ctx"], a["max_ctx"], a["B"],
+                a["n_q"], a["n_kv"], a["hd"], a["out"])
+
+    cases = [(dict(q=None), gf.GF_EINVAL), (dict(B=0), gf.GF_EINVAL), (dict(n_q=6, n_kv=4), gf.GF_EINVAL),
+             (dict(n_q=34, n_kv=2), gf.GF_EINVAL), (dict(hd=96), gf.GF_ENOTIMPL),
+             (dict(max_ctx=16 * 64 + 1), gf.GF_EINVAL), (dict(num_pages=0), gf.GF_EINVAL),
+             (dict(num_pages=1 << 26), gf.GF_EINVAL)]
+    for kw, code in cases:
+        for static in (False, True):
+            with pytest.raises(gf.GfError) as e:
+                if static:
+                    gf.gf_decode_attention_static(*call(**kw), None)
+                else:
+                    gf.gf_decode_attention(*call(**kw), ok["ws"], ok["ws_bytes"], None)
+            assert e.value.code == code, (kw, static)
+    with pytest.raises(gf.GfError) as e:
+        gf.gf_decode_attention(*call(), d, ws - 1, None)
+    assert e.value.code == gf.GF_EINVAL
+    # the fixed scratch of the allocation-free variant (16 MiB) bounds its problem size
+    big = dict(B=512, n_kv=8, max_ctx=16384, max_pages=256, num_pages=4096)
+    assert gf.gf_decode_attention_workspace(512, 8, 128, 16384) > 16 << 20
+    with pytest.raises(gf.GfError) as e:
+        gf.gf_decode_attention_static(*call(**big), None)
+    assert e.value.code == gf.GF_ECAPACITY
+
+
+def test_decode_attention_workspace_covers_every_chunking():
+    # partial results: 16 query rows x (head_dim outputs + max + sum) floats per (sequence, kv head, chunk);
+    # chunks are at least 256 keys, so the 256-key count bounds every plan
+    for B, n_kv, hd, ctx in [(1, 1, 64, 1), (4, 2, 128, 1000), (32, 4, 128, 6400), (128, 4, 128, 4096)]:
+        ws = gf.gf_decode_attention_workspace(B, n_kv, hd, ctx)
+        for chunk in (256, 512, 1024):
+            assert ws >= B * n_kv * -(-ctx // chunk) * 16 * (hd + 2) * 4
+        assert gf.gf_decode_attention_workspace(2 * B, n_kv, hd, ctx) == 2 * ws
+    assert gf.gf_decode_attention_workspace(0, 1, 128, 64) == 0
