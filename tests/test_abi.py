@@ -139,3 +139,19 @@ def test_decode_attention_workspace_covers_every_chunking():
             assert ws >= B * n_kv * -(-ctx // chunk) * 16 * (hd + 2) * 4
         assert gf.gf_decode_attention_workspace(2 * B, n_kv, hd, ctx) == 2 * ws
     assert gf.gf_decode_attention_workspace(0, 1, 128, 64) == 0
+
+
+def test_gemm_argument_validation_needs_no_gpu(lib):
+    d = ctypes.c_void_p(256)
+    ok = dict(A=d, W=d, M=32, N=256, K=128, out=d, ldo=256, mode=gf.GF_GEMM_STORE_F32, bn=0, splits=0, group_m=0)
+    cases = [dict(A=None), dict(out=None), dict(N=0), dict(K=32), dict(K=96), dict(N=48), dict(mode=5),
+             dict(mode=-1), dict(bn=96), dict(bn=32), dict(splits=2), dict(ldo=255),
+             dict(mode=gf.GF_GEMM_SWIGLU, ldo=127)]
+    for kw in cases:
+        a = dict(ok, **kw)
+        with pytest.raises(gf.GfError) as e:
+            gf.gf_gemm_bf16(a["A"], a["W"], a["M"], a["N"], a["K"], a["out"], a["ldo"], a["mode"], a["bn"],
+                            a["splits"], a["group_m"], None)
+        assert e.value.code == gf.GF_EINVAL, kw
+    # an empty product is a no-op (no device work)
+    gf.gf_gemm_bf16(d, d, 0, 256, 128, d, 256, gf.GF_GEMM_STORE_F32, 0, 0, 0, None)
