@@ -155,3 +155,13 @@ def test_gemm_argument_validation_needs_no_gpu(lib):
         assert e.value.code == gf.GF_EINVAL, kw
     # an empty product is a no-op (no device work)
     gf.gf_gemm_bf16(d, d, 0, 256, 128, d, 256, gf.GF_GEMM_STORE_F32, 0, 0, 0, None)
+
+
+def test_select_and_selftest_argument_validation_needs_no_gpu(lib):
+    d = ctypes.c_void_p(256)
+    for B, tau, p in [(0, 0.5, d), (1025, 0.5, d), (4, -0.1, d), (4, 1.5, d), (4, float("nan"), d), (4, 0.5, None)]:
+        with pytest.raises(gf.GfError) as e:
+            gf.gf_select(B, p, d, 1.5, tau, d, d, d, d, None)
+        assert e.value.code == gf.GF_EINVAL, (B, tau)
+    assert gf.gf_selftest_timeout(0, None) == gf.GF_EINVAL
+    assert gf.gf_selftest_timeout(2001, None) == gf.GF_EINVAL
