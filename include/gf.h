@@ -246,8 +246,10 @@ enum { GF_GEMM_STORE_F32 = 0, GF_GEMM_ADD_F32 = 1, GF_GEMM_ATOMIC_F32 = 2, GF_GE
        GF_GEMM_SWIGLU = 4 };
 int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
                  int32_t mode, int32_t bn, int32_t splits, int32_t group_m, void* stream);
-/* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16 or gf_decode_attention
- * launch gave up waiting. */
+/* Synchronise `stream`; GF_ETIMEOUT if a gf_gemm_bf16, gf_decode_attention or
+ * gf_selftest_timeout launch on the current device gave up waiting since the
+ * last call (the word it reads is then cleared).  The building blocks keep one
+ * such word per device (and CUDA context), made by their first call there. */
 int gf_gemm_status(void* stream);
 
 /* ---- planning queries (host arithmetic only: no device work, no GPU needed) --
@@ -308,18 +310,28 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
  *     exceed 16 MiB (16777216 bytes), else GF_ECAPACITY ("exceeds scratch")
  *     and nothing is enqueued;
  *   - the first call on a device, with that device current, looks up the
- *     array's device address (cudaGetSymbolAddress); make that first call
- *     before any stream capture;
+ *     array's device address (cudaGetSymbolAddress) for the current CUDA
+ *     context; make that first call before any stream capture.  A context
+ *     made later on the device (after cudaDeviceReset) gets the address
+ *     looked up again by its first call;
  *   - every call on a device shares the one array and it keeps the last
  *     call's contents, so calls whose work overlaps on the GPU (other streams,
  *     or other host threads) race and corrupt each other's results: order
- *     them.  A timeout word in the same fixed storage is cleared on `stream`
- *     at the start of each call.
+ *     them;
+ *   - a bounded wait that gives up (after 2 s) records a timeout in a word
+ *     of the same fixed storage and the call's output is then unspecified.
+ *     The word stays set, and later calls may give up early, until
+ *     gf_decode_attention_static_status reads and clears it: call that after
+ *     the work whose results you use.
  * It calls no cudaMalloc, cudaFree or other allocating routine. */
 int gf_decode_attention_static(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
                                const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len,
                                int32_t max_ctx, int32_t B, int32_t n_q, int32_t n_kv, int32_t head_dim, void* out,
                                void* stream);
+/* Failure report of gf_decode_attention_static on the current device:
+ * synchronises `stream`, then returns GF_ETIMEOUT (and clears the word) if a
+ * wait of any earlier call gave up, else GF_OK.  Allocates nothing. */
+int gf_decode_attention_static_status(void* stream);
 
 /* Failure detection self-test: launch a kernel whose bounded wait on a barrier
  * that nothing completes runs out after `limit_ms` (1..2000).  The kernel
@@ -327,6 +339,10 @@ int gf_decode_attention_static(const void* q, const void* k_cache, const void* v
  * returns GF_ETIMEOUT when the device reported it (GF_OK would mean the wait
  * did not run out).  The CUDA context stays usable. */
 int gf_selftest_timeout(uint32_t limit_ms, void* stream);
+/* The same self-test recording into the timeout word of
+ * gf_decode_attention_static: returns what gf_decode_attention_static_status
+ * then reports (GF_ETIMEOUT, with the word cleared again). */
+int gf_selftest_timeout_static(uint32_t limit_ms, void* stream);
 
 /* ---- measurement ------------------------------------------------------------
  * Kernel classes whose launches can be bracketed by CUDA events (on the

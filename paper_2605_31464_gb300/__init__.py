@@ -46,7 +46,8 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_forecast_batch_host", "gf_verdict", "gf_debug_capture", "gf_debug_read_kv", "gf_device_status",
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
-           "gf_decode_attention_static", "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select",
+           "gf_decode_attention_static", "gf_decode_attention_static_status", "gf_selftest_timeout_static",
+           "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select",
            "gf_forecast_batch_sampled", "gf_sample_tokens", "gf_plan_gemm", "gf_plan_decode_chunk"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
@@ -80,6 +81,8 @@ def load(path: str = LIB_PATH):
         "gf_sample_tokens": ([_c_i32, _p, _c_i64, _c_i32, ctypes.c_uint64, _c_i32, _c_f32, _p, _p], ctypes.c_int),
         "gf_free_pages": ([_p], _c_i64),
         "gf_selftest_timeout": ([ctypes.c_uint32, _p], ctypes.c_int),
+        "gf_selftest_timeout_static": ([ctypes.c_uint32, _p], ctypes.c_int),
+        "gf_decode_attention_static_status": ([_p], ctypes.c_int),
         "gf_select": ([_c_i32, _p, _p, _c_f32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_verdict": ([_c_i32, _p, _c_i64, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_debug_capture": ([_p, _c_i32, _c_i32, _p, _c_i64], ctypes.c_int),
@@ -272,6 +275,16 @@ def gf_decode_attention_static(q, k_cache, v_cache, num_pages, block_table, max_
     """gf_decode_attention with its scratch in the library's fixed device array (no allocation)."""
     _check(load().gf_decode_attention_static(q, k_cache, v_cache, num_pages, block_table, max_pages, ctx_len, max_ctx,
                                              B, n_q, n_kv, head_dim, out, stream))
+
+
+def gf_decode_attention_static_status(stream):
+    """Returns the status code (GF_OK, or GF_ETIMEOUT once after a timed-out wait) instead of raising."""
+    return int(load().gf_decode_attention_static_status(stream))
+
+
+def gf_selftest_timeout_static(limit_ms, stream):
+    """Returns the status code (GF_ETIMEOUT expected) instead of raising."""
+    return int(load().gf_selftest_timeout_static(limit_ms, stream))
 
 
 def decode_attention(q, k_cache, v_cache, block_table, ctx_len, max_ctx, n_q, n_kv, stream=None):

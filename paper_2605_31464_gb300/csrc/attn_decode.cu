@@ -345,16 +345,16 @@ __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
 template <int HD>
 static cudaError_t launch_hd(const CUtensorMap& tmK, const CUtensorMap& tmV, const DecodeAttnArgs& a, int B,
                              cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         DecodeCfg<HD>::SMEM);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  // the shared-memory limit is an attribute of the function in one device's context: set it once per context
+  static DeviceOnce configured;
+  cudaError_t e = configured.run([] {
+    return cudaFuncSetAttribute(attn_decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                DecodeCfg<HD>::SMEM);
+  });
+  if (e != cudaSuccess) return e;
   if (B == 0) return cudaSuccess;
   dim3 grid(a.max_splits, a.n_kv, B);
-  cudaError_t e = launch_pdl(attn_decode_kernel<HD>, grid, dim3(128), DecodeCfg<HD>::SMEM, s, tmK, tmV, a);
+  e = launch_pdl(attn_decode_kernel<HD>, grid, dim3(128), DecodeCfg<HD>::SMEM, s, tmK, tmV, a);
   if (e != cudaSuccess) return e;
   return launch_pdl(attn_combine_kernel<HD>, dim3(B * a.n_q), dim3(HD), 0, s, a);
 }
@@ -376,14 +376,57 @@ cudaError_t launch_attn_decode(int hd, const CUtensorMap& tmK, const CUtensorMap
 namespace {
 constexpr size_t kStaticScratchBytes = size_t(16) << 20;  // 16 MiB, held by every GPU that loads the library
 constexpr int kMaxDevices = 64;
+// Device addresses of the arrays, looked up once per device and CUDA context (ctx = its unique id).
+struct StaticAddrs {
+  uint64_t ctx = 0;
+  void* scratch = nullptr;
+  int* err = nullptr;
+};
 std::mutex g_static_mu;
-bool g_static_ready[kMaxDevices];
-void* g_static_scratch_ptr[kMaxDevices];
-int* g_static_err_ptr[kMaxDevices];
+StaticAddrs g_static[kMaxDevices];
 }  // namespace
 
 static __device__ __align__(256) unsigned char g_static_scratch[kStaticScratchBytes];
+// Timeout word of the allocation-free entry point: set by a bounded wait that gave up, cleared only by
+// gf_decode_attention_static_status (zero when the module is loaded).
 static __device__ __align__(256) int g_static_err;
+
+// Set-up, with the device current: the device addresses of the two arrays.  In host code their names
+// stand for host-side shadows, not device memory, so the kernels get the addresses
+// cudaGetSymbolAddress reports.  The lookup runs on the first call in each context of a device (it
+// may load this module there, which is why the first call must not fall inside a stream capture) and
+// again in a context made later, after cudaDeviceReset; it allocates nothing itself.
+static int static_addrs(void** scratch, int** err) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    gf::set_error_short("no CUDA device");
+    return GF_ECUDA;
+  }
+  if (dev < 0 || dev >= kMaxDevices) {
+    gf::set_error_short("too many GPUs");
+    return GF_ENOTIMPL;
+  }
+  const uint64_t ctx = gf::current_context_id();
+  std::lock_guard<std::mutex> lock(g_static_mu);
+  StaticAddrs& a = g_static[dev];
+  if (ctx == 0 || a.ctx != ctx || !a.scratch) {
+    void* sp = nullptr;
+    void* ep = nullptr;
+    if (cudaGetSymbolAddress(&sp, g_static_scratch) != cudaSuccess ||
+        cudaGetSymbolAddress(&ep, g_static_err) != cudaSuccess || !sp || !ep) {
+      cudaGetLastError();
+      gf::set_error_short("symbol lookup");
+      return GF_ECUDA;
+    }
+    a.ctx = ctx;
+    a.scratch = sp;
+    a.err = reinterpret_cast<int*>(ep);
+  }
+  *scratch = a.scratch;
+  *err = a.err;
+  return GF_OK;
+}
 
 extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, const void* v_cache, int64_t num_pages,
                                           const int32_t* block_table, int32_t max_pages, const int32_t* ctx_len,
@@ -404,40 +447,14 @@ extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, co
     gf::set_error_short("exceeds scratch");
     return GF_ECAPACITY;
   }
-  int dev = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess) {
-    gf::set_error_short("no CUDA device");
-    return GF_ECUDA;
-  }
-  if (dev < 0 || dev >= kMaxDevices) {
-    gf::set_error_short("too many GPUs");
-    return GF_ENOTIMPL;
-  }
-  {
-    // First call on this device: look up the device addresses of the arrays
-    // (host code cannot use their names as device pointers).
-    std::lock_guard<std::mutex> lock(g_static_mu);
-    if (!g_static_ready[dev]) {
-      void* scratch = nullptr;
-      void* err = nullptr;
-      if (cudaGetSymbolAddress(&scratch, g_static_scratch) != cudaSuccess ||
-          cudaGetSymbolAddress(&err, g_static_err) != cudaSuccess) {
-        cudaGetLastError();
-        gf::set_error_short("symbol lookup");
-        return GF_ECUDA;
-      }
-      g_static_scratch_ptr[dev] = scratch;
-      g_static_err_ptr[dev] = reinterpret_cast<int*>(err);
-      g_static_ready[dev] = true;
-    }
-  }
+  void* scratch = nullptr;
+  int* err = nullptr;
+  const int rc = static_addrs(&scratch, &err);
+  if (rc != GF_OK) return rc;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  // The timeout word must start at zero: a word left set by an earlier call
-  // would make this call's waits give up at once.
-  if (cudaMemsetAsync(g_static_err_ptr[dev], 0, sizeof(int), s) != cudaSuccess) {
-    gf::set_error_short("memset failed");
-    return GF_ECUDA;
-  }
+  // Nothing in the scratch needs clearing: every partial the merge reads is written first by this
+  // call.  The timeout word is not cleared here, so that a timeout stays visible to
+  // gf_decode_attention_static_status however many calls follow it.
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
   if (gf::encode_kv_map(&tk, k_cache, head_dim, rows) ||
@@ -460,15 +477,59 @@ extern "C" int gf_decode_attention_static(const void* q, const void* k_cache, co
   da.layer_vrow0 = 0;
   da.chunk = 256;
   da.max_splits = (max_ctx + 255) / 256;
-  da.part_o = reinterpret_cast<float*>(g_static_scratch_ptr[dev]);
+  da.part_o = reinterpret_cast<float*>(scratch);
   da.part_ml = da.part_o + (size_t)B * n_kv * da.max_splits * 16 * head_dim;
   da.out = reinterpret_cast<gf::bf16*>(out);
   da.ldo = (int64_t)n_q * head_dim;
   da.scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
-  da.err = g_static_err_ptr[dev];
+  da.err = err;
   if (gf::launch_attn_decode(head_dim, tk, tv, da, B, s) != cudaSuccess) {
+    cudaGetLastError();
     gf::set_error_short("launch failed");
     return GF_ECUDA;
   }
   return GF_OK;
+}
+
+extern "C" int gf_decode_attention_static_status(void* stream) {
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    gf::set_error_short("sync failed");
+    return GF_ECUDA;
+  }
+  void* scratch = nullptr;
+  int* err = nullptr;
+  const int rc = static_addrs(&scratch, &err);
+  if (rc != GF_OK) return rc;
+  int h = 0;
+  if (cudaMemcpyAsync(&h, err, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+      cudaMemsetAsync(err, 0, sizeof(int), s) != cudaSuccess || cudaStreamSynchronize(s) != cudaSuccess) {
+    cudaGetLastError();
+    gf::set_error_short("status read");
+    return GF_ECUDA;
+  }
+  if (h == gf::kErrTimeout) {
+    gf::set_error_short("wait timed out");
+    return GF_ETIMEOUT;
+  }
+  return GF_OK;
+}
+
+extern "C" int gf_selftest_timeout_static(uint32_t limit_ms, void* stream) {
+  if (limit_ms < 1 || limit_ms > 2000) {
+    gf::set_error_short("bad limit");
+    return GF_EINVAL;
+  }
+  void* scratch = nullptr;
+  int* err = nullptr;
+  const int rc = static_addrs(&scratch, &err);
+  if (rc != GF_OK) return rc;
+  if (gf::launch_timeout_probe((uint64_t)limit_ms * 1000000ull, err, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess) {
+    cudaGetLastError();
+    gf::set_error_short("launch failed");
+    return GF_ECUDA;
+  }
+  return gf_decode_attention_static_status(stream);
 }

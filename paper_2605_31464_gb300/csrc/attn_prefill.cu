@@ -354,13 +354,13 @@ __global__ void __launch_bounds__(384, 1) attn_prefill_tc_kernel(const __grid_co
 template <int HD>
 static cudaError_t launch_hd(const CUtensorMap& tmQ, const CUtensorMap& tmK, const CUtensorMap& tmV,
                              const PrefillAttnArgs& a, int n_items, cudaStream_t s) {
-  static bool configured = false;
-  if (!configured) {
-    cudaError_t e = cudaFuncSetAttribute(attn_prefill_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         FaCfg<HD>::SMEM);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  // the shared-memory limit is an attribute of the function in one device's context: set it once per context
+  static DeviceOnce configured;
+  const cudaError_t e = configured.run([] {
+    return cudaFuncSetAttribute(attn_prefill_tc_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                FaCfg<HD>::SMEM);
+  });
+  if (e != cudaSuccess) return e;
   const int64_t grid = (int64_t)n_items * a.n_q;
   if (grid == 0) return cudaSuccess;
   return launch_pdl(attn_prefill_tc_kernel<HD>, dim3((unsigned)grid), dim3(FaCfg<HD>::THREADS), FaCfg<HD>::SMEM, s,

@@ -15,14 +15,13 @@ int gemm_smem_bytes(int bn) {
 template <int BN, int MODE, bool SWAP>
 static cudaError_t launch_one(const CUtensorMap& tmA, const CUtensorMap& tmB, const GemmArgs& p, int grid,
                               cudaStream_t s) {
-  static bool configured = false;
+  // the shared-memory limit is an attribute of the function in one device's context: set it once per context
+  static DeviceOnce configured;
   auto kern = gemm_tc_kernel<BN, MODE, SWAP>;
-  if (!configured) {
-    cudaError_t e =
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN, SWAP>::SMEM_BYTES);
-    if (e != cudaSuccess) return e;
-    configured = true;
-  }
+  const cudaError_t e = configured.run([&] {
+    return cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, GemmCfg<BN, SWAP>::SMEM_BYTES);
+  });
+  if (e != cudaSuccess) return e;
   return launch_pdl(kern, dim3(grid), dim3(GemmCfg<BN, SWAP>::THREADS), GemmCfg<BN, SWAP>::SMEM_BYTES, s, tmA, tmB,
                     p);
 }

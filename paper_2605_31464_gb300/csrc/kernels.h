@@ -6,6 +6,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "sampling.cuh"
 
 namespace gf {
@@ -43,6 +45,30 @@ inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, siz
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
 }
+
+// A set-up step that holds for one CUDA context, such as raising a kernel's shared-memory limit
+// (an attribute of the function as loaded in the current device's context): run() calls `f` the
+// first time it is reached in each context, and does nothing later in the same context.  Contexts
+// are told apart per device (up to 64 devices; beyond that `f` runs every time) by
+// current_context_id(), so a context made again after cudaDeviceReset runs `f` again.  Several host
+// threads may call run() at once; `f` must then be safe to repeat.
+// current_context_id (runtime.cu): the unique id (cuCtxGetId) of the calling thread's current CUDA
+// context, 0 if it cannot be read; a context made after cudaDeviceReset gets a new id.
+uint64_t current_context_id();
+struct DeviceOnce {
+  std::atomic<uint64_t> ctx[64] = {};
+  template <typename F>
+  cudaError_t run(F&& f) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t id = current_context_id();
+    if (dev >= 0 && dev < 64 && id != 0 && ctx[dev].load(std::memory_order_acquire) == id) return cudaSuccess;
+    e = f();
+    if (e == cudaSuccess && dev >= 0 && dev < 64 && id != 0) ctx[dev].store(id, std::memory_order_release);
+    return e;
+  }
+};
 
 // ------------------------------------------------------------------ GEMM
 // C[M,N] (op)= A[M,K] . B[N,K]^T ; mode is a GemmMode.  tmA/tmB are 2D

@@ -7,6 +7,7 @@
 #include <cstdio>
 #include <cstring>
 #include <map>
+#include <mutex>
 #include <string>
 #include <tuple>
 #include <vector>
@@ -973,6 +974,29 @@ int encode_vt_map(CUtensorMap* m, const void* base, int hd, uint64_t rows) {
 }
 // Record a message of at most 15 characters (kept in the string's inline buffer, so nothing is allocated).
 void set_error_short(const char* msg) { g_err = msg; }
+
+uint64_t current_context_id() {
+  typedef CUresult (*GetCurrentFn)(CUcontext*);
+  typedef CUresult (*GetIdFn)(CUcontext, unsigned long long*);
+  static GetCurrentFn get_current = nullptr;
+  static GetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<GetCurrentFn>(p);
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<GetIdFn>(p);
+  });
+  if (!get_current || !get_id) return 0;
+  CUcontext c = nullptr;
+  unsigned long long id = 0;
+  if (get_current(&c) != CUDA_SUCCESS || !c || get_id(c, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
 }  // namespace gf
 
 // =====================================================================================================
@@ -1395,7 +1419,48 @@ int gf_forecast_batch_host(gf_model* m, int32_t B, const int32_t* inc_ids, const
   return GF_OK;
 }
 
-static int* g_gemm_err = nullptr;
+// Timeout word of the building blocks (gf_gemm_bf16, gf_decode_attention, gf_selftest_timeout): one
+// per device and CUDA context, allocated the first time a building block runs there.
+namespace {
+struct ErrWord {
+  uint64_t ctx = 0;
+  int* ptr = nullptr;
+};
+std::mutex g_err_mu;
+ErrWord g_err_words[64];
+
+// *out = the current device's word (nullptr when `create` is false and none exists yet); GF_OK or
+// the reason it cannot be had.
+int block_err_word(bool create, int** out) {
+  *out = nullptr;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) {
+    cudaGetLastError();
+    return fail(GF_ECUDA, "no CUDA device");
+  }
+  if (dev < 0 || dev >= 64) return fail(GF_ENOTIMPL, "device ordinal %d: the building blocks serve devices 0..63", dev);
+  const uint64_t ctx = gf::current_context_id();
+  std::lock_guard<std::mutex> lock(g_err_mu);
+  ErrWord& w = g_err_words[dev];
+  if (w.ptr && w.ctx == ctx) {
+    *out = w.ptr;
+    return GF_OK;
+  }
+  if (!create) return GF_OK;
+  // a word of an earlier context of this device went away with that context (cudaDeviceReset)
+  w.ptr = nullptr;
+  int* p = nullptr;
+  if (cudaMalloc(&p, sizeof(int)) != cudaSuccess || cudaMemset(p, 0, sizeof(int)) != cudaSuccess) {
+    cudaGetLastError();
+    if (p) cudaFree(p);
+    return fail(GF_ENOMEM, "error word allocation failed");
+  }
+  w.ptr = p;
+  w.ctx = ctx;
+  *out = p;
+  return GF_OK;
+}
+}  // namespace
 
 int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, void* out, int64_t ldo,
                  int32_t mode, int32_t bn, int32_t splits, int32_t group_m, void* stream) {
@@ -1408,10 +1473,8 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   if (ldo < (mode == GF_GEMM_SWIGLU ? N / 2 : N)) return fail(GF_EINVAL, "ldo too small");
   if (M == 0) return GF_OK;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (!g_gemm_err) {
-    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
-    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
-  }
+  int* err = nullptr;
+  TRY(block_err_word(true, &err));
   int dev = 0, sms = 0;
   CU(cudaGetDevice(&dev));
   CU(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev));
@@ -1426,11 +1489,11 @@ int gf_gemm_bf16(const void* A, const void* W, int32_t M, int32_t N, int32_t K, 
   if (swap) {
     TRY(make_map(&ta, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, 128));
     TRY(make_map(&tb, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, (uint32_t)bn));
-    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m, true));
+    CU(gf::launch_gemm(ta, tb, N, M, K, out, ldo, mode, bn, splits, sms, err, s, group_m, true));
   } else {
     TRY(make_map(&ta, A, (uint64_t)K, (uint64_t)M, (uint64_t)K * 2, 64, 128));
     TRY(make_map(&tb, W, (uint64_t)K, (uint64_t)N, (uint64_t)K * 2, 64, (uint32_t)bn));
-    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, g_gemm_err, s, group_m));
+    CU(gf::launch_gemm(ta, tb, M, N, K, out, ldo, mode, bn, splits, sms, err, s, group_m));
   }
   return GF_OK;
 }
@@ -1460,12 +1523,16 @@ int32_t gf_plan_decode_chunk(int32_t B, int32_t n_kv, int32_t max_ctx, int32_t s
 }
 
 int gf_gemm_status(void* stream) {
-  CU(cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)));
-  if (!g_gemm_err) return GF_OK;  // shared by gf_gemm_bf16 and gf_decode_attention
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  CU(cudaStreamSynchronize(s));
+  int* err = nullptr;  // shared by gf_gemm_bf16, gf_decode_attention and gf_selftest_timeout
+  TRY(block_err_word(false, &err));
+  if (!err) return GF_OK;  // no building block has run in this context
   int h = 0;
-  CU(cudaMemcpy(&h, g_gemm_err, sizeof(int), cudaMemcpyDeviceToHost));
-  CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
-  if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a GEMM wait timed out");
+  CU(cudaMemcpyAsync(&h, err, sizeof(int), cudaMemcpyDeviceToHost, s));
+  CU(cudaMemsetAsync(err, 0, sizeof(int), s));
+  CU(cudaStreamSynchronize(s));
+  if (h == gf::kErrTimeout) return fail(GF_ETIMEOUT, "a device-side wait timed out");
   return GF_OK;
 }
 
@@ -1487,10 +1554,8 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   if (num_pages < 1 || num_pages * n_kv * 64 >= ((int64_t)1 << 31)) return fail(GF_EINVAL, "bad page count");
   if (workspace_bytes < gf_decode_attention_workspace(B, n_kv, head_dim, max_ctx))
     return fail(GF_EINVAL, "workspace smaller than gf_decode_attention_workspace()");
-  if (!g_gemm_err) {
-    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
-    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
-  }
+  int* err = nullptr;
+  TRY(block_err_word(true, &err));
   CUtensorMap tk, tv;
   const uint64_t rows = (uint64_t)num_pages * n_kv * 64;
   TRY(make_map(&tk, k_cache, head_dim, rows, head_dim * 2, 64, 64));
@@ -1518,7 +1583,7 @@ int gf_decode_attention(const void* q, const void* k_cache, const void* v_cache,
   da.out = reinterpret_cast<bf16*>(out);
   da.ldo = (int64_t)n_q * head_dim;
   da.scale_log2 = 1.4426950408889634f / sqrtf((float)head_dim);
-  da.err = g_gemm_err;
+  da.err = err;
   CU(gf::launch_attn_decode(head_dim, tk, tv, da, B, reinterpret_cast<cudaStream_t>(stream)));
   return GF_OK;
 }
@@ -1536,11 +1601,9 @@ int gf_select(int32_t B, const float* p, const float* m_bins, float x_cut, float
 int gf_selftest_timeout(uint32_t limit_ms, void* stream) {
   if (limit_ms < 1 || limit_ms > 2000) return fail(GF_EINVAL, "limit_ms outside 1..2000");
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  if (!g_gemm_err) {
-    CU(cudaMalloc(&g_gemm_err, sizeof(int)));
-    CU(cudaMemset(g_gemm_err, 0, sizeof(int)));
-  }
-  CU(gf::launch_timeout_probe((uint64_t)limit_ms * 1000000ull, g_gemm_err, s));
+  int* err = nullptr;
+  TRY(block_err_word(true, &err));
+  CU(gf::launch_timeout_probe((uint64_t)limit_ms * 1000000ull, err, s));
   return gf_gemm_status(stream);
 }
 

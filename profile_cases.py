@@ -1,9 +1,9 @@
 """Run one hot-path kernel at a chosen workload shape (for profilers).
 
-    python -m paper_2605_31464_gb300.profile_cases gemm --M 8192 --N 37888 --K 3584 --mode swiglu
-    python -m paper_2605_31464_gb300.profile_cases decode_attn --B 128 --ctx 3072 --n_q 28 --n_kv 4
-    python -m paper_2605_31464_gb300.profile_cases prefill --workload 7b_prefill --batch 2 --layers 2
-    python -m paper_2605_31464_gb300.profile_cases forecast --workload 7b_prefill --layers 4 --n_decode 16
+    python profile_cases.py gemm --M 8192 --N 37888 --K 3584 --mode swiglu
+    python profile_cases.py decode_attn --B 128 --ctx 3072 --n_q 28 --n_kv 4
+    python profile_cases.py prefill --workload 7b_prefill --batch 2 --layers 2
+    python profile_cases.py forecast --workload 7b_prefill --layers 4 --n_decode 16
 
 Each case launches the kernel `--repeat` times on synthetic data through
 the C ABI and prints the mean CUDA-event time and the algorithmic rate.
@@ -153,7 +153,7 @@ def _forecast(a):
 
 
 def main(argv=None):
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    root = os.path.dirname(os.path.abspath(__file__))
     if root not in sys.path:
         sys.path.insert(0, root)
     ap = argparse.ArgumentParser()

@@ -56,6 +56,31 @@ def check_logits(gpu: np.ndarray, ref: np.ndarray, what: str = "logits"):
     return float(err.max())
 
 
+# Full-depth end-to-end logits (28 layers from token ids): the per-element bound above holds for all
+# but a few of the 151,936 logits of a 1.5B-class item.  The bf16 rounding of the activations is what
+# exceeds it: the float64 oracle with bf16 rounding at the GPU path's rounding points (GEMM inputs,
+# rotated q/k, cached v, softmax numerators, attention output, SwiGLU output) misses the bound on 3 of
+# 151,936 prompt logits of 1p5b item 5, by up to 1.10x.  So at full depth at most DEEP_FRAC of the
+# logits may exceed the bound, none by more than DEEP_RATIO, and the mean error must stay within
+# DEEP_MEAN (that emulation: 0.0059).
+DEEP_FRAC = 1e-4
+DEEP_RATIO = 1.5
+DEEP_MEAN = 0.25 * LOGIT_ATOL
+
+
+def check_logits_deep(gpu: np.ndarray, ref: np.ndarray, what: str = "logits"):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    err = np.abs(gpu - ref)
+    ratio = err / (LOGIT_ATOL + LOGIT_RTOL * np.abs(ref))
+    n_out = int((ratio > 1).sum())
+    msg = (f"{what}: mean err {err.mean():.4g}, max err {err.max():.4g}, {n_out} of {err.size} beyond the "
+           f"per-element bound, worst {ratio.max():.3f}x")
+    assert err.mean() <= DEEP_MEAN, msg
+    assert n_out <= DEEP_FRAC * err.size, msg
+    assert ratio.max() <= DEEP_RATIO, msg
+    return msg
+
+
 def greedy_agrees(gpu_tok: int, ref_logits: np.ndarray) -> bool:
     """GPU arg max equals the oracle's, or the oracle's top-2 gap is within the tie band."""
     order = np.argsort(-ref_logits, kind="stable")
