@@ -25,6 +25,13 @@ namespace gf {
 #define GF_DECODE_STAGES 2
 #endif
 
+// Keys per split when the splits adapt to the context (DecodeAttnArgs::chunk == 0): the sequence's
+// pages shared as evenly as whole pages allow among the `splits` CTAs of its row of the grid.
+__device__ __forceinline__ int decode_chunk_of(int ctx, int splits) {
+  const int pages = (ctx + 63) >> 6;
+  return ((pages + splits - 1) / splits) * 64;
+}
+
 template <int HD>
 struct DecodeCfg {
   static constexpr int STAGES = GF_DECODE_STAGES;   // pages (K + V^T) in flight per CTA
@@ -56,9 +63,10 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int slot = a.handles ? a.handles[b] : b;
   const int pos = a.seq_len[slot];  // the new token's position (fused step)
   const int ctx = min(pos + a.ctx_bias, a.max_ctx);
-  const int k0 = split * a.chunk;
+  const int chunk = a.chunk > 0 ? a.chunk : decode_chunk_of(ctx, a.max_splits);
+  const int k0 = split * chunk;
   if (k0 >= ctx) return;
-  const int k1 = min(k0 + a.chunk, ctx);
+  const int k1 = min(k0 + chunk, ctx);
   const int p0 = k0 >> 6;
   const int n_pages = ((k1 - 1) >> 6) - p0 + 1;
   const int G = a.n_q / a.n_kv;
@@ -314,7 +322,8 @@ __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
   const int G = a.n_q / a.n_kv;
   const int kvh = h / G, r = h % G;
   const int ctx = min(a.seq_len[a.handles ? a.handles[b] : b] + a.ctx_bias, a.max_ctx);
-  const int n_splits = ctx > 0 ? min((ctx + a.chunk - 1) / a.chunk, a.max_splits) : 0;
+  const int chunk = a.chunk > 0 ? a.chunk : decode_chunk_of(ctx, a.max_splits);
+  const int n_splits = ctx > 0 ? min((ctx + chunk - 1) / chunk, a.max_splits) : 0;
   const int64_t base = ((int64_t)b * a.n_kv + kvh) * a.max_splits;
   float M = -INFINITY;
   for (int s = 0; s < n_splits; ++s) M = fmaxf(M, a.part_ml[((base + s) * 16 + r) * 2]);
