@@ -228,6 +228,25 @@ int gf_verdict(int32_t B, const float* logits, int64_t ld, const int32_t* verdic
 int gf_select(int32_t B, const float* p, const float* m_bins, float x_cut, float tau_disc, float* s_hat,
               int32_t* order, float* disc, uint8_t* disc_pred, void* stream);
 
+/* ---- evaluation of 8-bin forecasts (host arithmetic only; no device work, no GPU needed) ----
+ * gf_speedup_bin: the bin 1..8 of a measured speedup S (Table tab:speedup-bins, upper edges
+ * inclusive: S <= 0.25, (0.25,0.5], (0.5,0.71], (0.71,1], (1,1.41], (1.41,2], (2,4], > 4).
+ * gf_score_forecasts: the scores of n forecasts p [n*8] (host, row i = bins 1..8 of candidate i)
+ * against the measured speedups S [n] (host, > 0), with bin representatives m_bins [8]:
+ *   scores[0] = speedup recovered (Sec. 3.1): 100/|C| sum_{c in C} max_{i in Top_c} S_i / max_i S_i,
+ *               C = {1, 5, 10, 25, 50} %, Top_c = the first ceil(c n / 100) (at least one) candidates
+ *               by decreasing sum_b p_ib m_b, lower index first on ties;
+ *   scores[1] = expected calibration error (Sec. 3.1): ten equal-width buckets of q_i = max_b p_ib,
+ *               (0, 0.1] ... (0.9, 1] (0 in the first), accuracy = predicted bin (arg max, lowest bin
+ *               on ties) equal to the measured bin;
+ *   scores[2] = forecast error (Sec. 3.1): mean |m_{predicted bin} - S_i|;
+ *   scores[3] = mean Brier score (Sec. 2.2): 1/2 sum_b (p_ib - 1[b = y_i])^2, y_i the measured bin;
+ *   scores[4] = mean CRPS (Sec. 2.2): 1/7 sum_{k=1..7} (F_ik - 1[y_i <= k])^2, F the cumulative p.
+ * scores: host double[5].  GF_EINVAL for n < 1, a null pointer, a negative or non-finite p or a
+ * non-positive speedup. */
+int gf_speedup_bin(double S);
+int gf_score_forecasts(int32_t n, const double* p, const double* S, const double* m_bins, double* scores);
+
 /* ---- building blocks --------------------------------------------------------
  * The dense contraction every projection of the forward pass uses, exposed on
  * its own: out[M,N] (op)= A[M,K] . W[N,K]^T on the tcgen05 tensor cores.

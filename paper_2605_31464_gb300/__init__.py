@@ -47,7 +47,7 @@ EXPORTS = ["gf_create", "gf_destroy", "gf_prefill", "gf_decode_step", "gf_releas
            "gf_launch_count", "gf_last_error", "gf_gemm_bf16", "gf_gemm_status", "gf_profile_enable",
            "gf_profile_read", "gf_decode_attention", "gf_decode_attention_workspace",
            "gf_decode_attention_static", "gf_decode_attention_static_status", "gf_selftest_timeout_static",
-           "gf_forecast_batch_shared", "gf_free_pages", "gf_selftest_timeout", "gf_select",
+           "gf_forecast_batch_shared", "gf_speedup_bin", "gf_score_forecasts", "gf_free_pages", "gf_selftest_timeout", "gf_select",
            "gf_forecast_batch_sampled", "gf_sample_tokens", "gf_plan_gemm", "gf_plan_decode_chunk"]
 
 GF_GEMM_STORE_F32, GF_GEMM_ADD_F32, GF_GEMM_ATOMIC_F32, GF_GEMM_STORE_BF16, GF_GEMM_SWIGLU = range(5)
@@ -82,6 +82,8 @@ def load(path: str = LIB_PATH):
         "gf_free_pages": ([_p], _c_i64),
         "gf_selftest_timeout": ([ctypes.c_uint32, _p], ctypes.c_int),
         "gf_selftest_timeout_static": ([ctypes.c_uint32, _p], ctypes.c_int),
+        "gf_speedup_bin": ([ctypes.c_double], ctypes.c_int),
+        "gf_score_forecasts": ([_c_i32, _p, _p, _p, _p], ctypes.c_int),
         "gf_decode_attention_static_status": ([_p], ctypes.c_int),
         "gf_select": ([_c_i32, _p, _p, _c_f32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
         "gf_verdict": ([_c_i32, _p, _c_i64, _p, _c_i32, _c_f32, _p, _p, _p, _p, _p], ctypes.c_int),
@@ -207,6 +209,24 @@ def select(p, m_bins, x_cut, tau_disc, stream=None):
 def gf_selftest_timeout(limit_ms, stream):
     """Returns the status code (GF_ETIMEOUT expected) instead of raising."""
     return int(load().gf_selftest_timeout(limit_ms, stream))
+
+
+def gf_speedup_bin(S) -> int:
+    """Bin 1..8 of a measured speedup (host arithmetic only; needs no GPU)."""
+    return int(load().gf_speedup_bin(float(S)))
+
+
+def score_forecasts(p, S, m_bins) -> dict:
+    """Speedup recovered, ECE, forecast error, mean Brier and CRPS of 8-bin forecasts p [n, 8] against
+    measured speedups S [n] (host arithmetic only; needs no GPU)."""
+    p = np.ascontiguousarray(np.asarray(p, dtype=np.float64))
+    S = np.ascontiguousarray(np.asarray(S, dtype=np.float64))
+    m = np.ascontiguousarray(np.asarray(m_bins, dtype=np.float64))
+    if p.ndim != 2 or p.shape[1] != 8 or S.shape != (p.shape[0],) or m.shape != (8,):
+        raise ValueError("p must be [n, 8], S [n] and m_bins [8]")
+    out = np.zeros(5, dtype=np.float64)
+    _check(load().gf_score_forecasts(p.shape[0], _ptr(p), _ptr(S), _ptr(m), _ptr(out)))
+    return dict(recovered=out[0], ece=out[1], forecast_error=out[2], brier=out[3], crps=out[4])
 
 
 def gf_free_pages(model) -> int:
