@@ -21,16 +21,12 @@
 
 namespace gf {
 
+// Most pages one decode-attention CTA may read (its page numbers are kept in shared memory).
+constexpr int kDecodeMaxChunkPages = 64;
+
 #ifndef GF_DECODE_STAGES
 #define GF_DECODE_STAGES 2
 #endif
-
-// Keys per split when the splits adapt to the context (DecodeAttnArgs::chunk == 0): the sequence's
-// pages shared as evenly as whole pages allow among the `splits` CTAs of its row of the grid.
-__device__ __forceinline__ int decode_chunk_of(int ctx, int splits) {
-  const int pages = (ctx + 63) >> 6;
-  return ((pages + splits - 1) / splits) * 64;
-}
 
 template <int HD>
 struct DecodeCfg {
@@ -39,8 +35,10 @@ struct DecodeCfg {
   static constexpr int PAGE_HALF = 64 * 128;        // one 64-column half of a K page
   static constexpr int PAGE_BYTES = 64 * HD * 2;    // one page of K (or V^T) for one head
   static constexpr int Q_BYTES = 16 * HD * 2;
-  // smem: Q [HALVES][16][128 B] | K[STAGES] | V[STAGES] | barriers; the K/V area is reused to combine warps
+  // smem: Q [HALVES][16][128 B] | K[STAGES] | V[STAGES] | barriers | the chunk's page numbers [pg_cap];
+  // the K/V area is reused to combine warps
   static constexpr int SMEM = 1024 + Q_BYTES + 2 * STAGES * PAGE_BYTES + 8 * STAGES;
+  static constexpr int smem(int pg_cap) { return SMEM + 4 * pg_cap; }
 };
 
 template <int HD>
@@ -56,6 +54,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   uint8_t* sK = sQ + C::Q_BYTES;
   uint8_t* sV = sK + C::STAGES * C::PAGE_BYTES;
   uint64_t* bar = reinterpret_cast<uint64_t*>(sV + C::STAGES * C::PAGE_BYTES);  // [STAGES]
+  int* spage = reinterpret_cast<int*>(bar + C::STAGES);                           // [pg_cap]
 
   const int split = blockIdx.x;
   const int kvh = blockIdx.y;
@@ -63,10 +62,9 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int slot = a.handles ? a.handles[b] : b;
   const int pos = a.seq_len[slot];  // the new token's position (fused step)
   const int ctx = min(pos + a.ctx_bias, a.max_ctx);
-  const int chunk = a.chunk > 0 ? a.chunk : decode_chunk_of(ctx, a.max_splits);
-  const int k0 = split * chunk;
+  const int k0 = split * a.chunk;
   if (k0 >= ctx) return;
-  const int k1 = min(k0 + chunk, ctx);
+  const int k1 = min(k0 + a.chunk, ctx);
   const int p0 = k0 >> 6;
   const int n_pages = ((k1 - 1) >> 6) - p0 + 1;
   const int G = a.n_q / a.n_kv;
@@ -74,9 +72,9 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
   const int lane = threadIdx.x & 31;
   const int32_t* pages = a.block_table + (int64_t)slot * a.max_pages;
 
-  auto issue = [&](int i) {
+  auto issue = [&](int i, int page) {
     const int buf = i % C::STAGES;
-    const int64_t pg = (int64_t)pages[p0 + i] * a.n_kv + kvh;
+    const int64_t pg = (int64_t)page * a.n_kv + kvh;
     mbar_arrive_expect_tx(&bar[buf], 2 * C::PAGE_BYTES);
 #pragma unroll
     for (int h = 0; h < C::HALVES; ++h)
@@ -95,8 +93,10 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
     for (int i = 0; i < C::STAGES; ++i) mbar_init(&bar[i], 1);
     fence_mbar_init();
     fence_async_smem();
-    for (int i = 0; i < first_copies - (defer_last ? 1 : 0); ++i) issue(i);
+    for (int i = 0; i < first_copies - (defer_last ? 1 : 0); ++i) issue(i, pages[p0 + i]);
   }
+  // the chunk's page numbers, so that a later copy does not wait for a load of its page number
+  for (int i = threadIdx.x; i < n_pages; i += blockDim.x) spage[i] = pages[p0 + i];
   if (fused) {
     // rotated queries of this group as bf16, swizzled like TMA; rows G..15 are zero.  Each thread
     // handles up to four (row, pair) items, all loads first.
@@ -154,7 +154,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
     }
   }
   __syncthreads();
-  if (defer_last && threadIdx.x == 0) issue(n_pages - 1);
+  if (defer_last && threadIdx.x == 0) issue(n_pages - 1, spage[n_pages - 1]);
 
   uint32_t qa[HD / 16][4];
   {
@@ -256,7 +256,7 @@ __global__ void __launch_bounds__(128) attn_decode_kernel(const __grid_constant_
       mma_bf16_16816(o[2 * dp + 1], pa, b2, b3);
     }
     __syncthreads();
-    if (threadIdx.x == 0 && i + C::STAGES < n_pages) issue(i + C::STAGES);
+    if (threadIdx.x == 0 && i + C::STAGES < n_pages) issue(i + C::STAGES, spage[i + C::STAGES]);
   }
 
   if (!ok) {
@@ -322,8 +322,7 @@ __global__ void attn_combine_kernel(const DecodeAttnArgs a) {
   const int G = a.n_q / a.n_kv;
   const int kvh = h / G, r = h % G;
   const int ctx = min(a.seq_len[a.handles ? a.handles[b] : b] + a.ctx_bias, a.max_ctx);
-  const int chunk = a.chunk > 0 ? a.chunk : decode_chunk_of(ctx, a.max_splits);
-  const int n_splits = ctx > 0 ? min((ctx + chunk - 1) / chunk, a.max_splits) : 0;
+  const int n_splits = ctx > 0 ? min((ctx + a.chunk - 1) / a.chunk, a.max_splits) : 0;
   const int64_t base = ((int64_t)b * a.n_kv + kvh) * a.max_splits;
   float M = -INFINITY;
   for (int s = 0; s < n_splits; ++s) M = fmaxf(M, a.part_ml[((base + s) * 16 + r) * 2]);
@@ -358,12 +357,14 @@ static cudaError_t launch_hd(const CUtensorMap& tmK, const CUtensorMap& tmV, con
   static DeviceOnce configured;
   cudaError_t e = configured.run([] {
     return cudaFuncSetAttribute(attn_decode_kernel<HD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                DecodeCfg<HD>::SMEM);
+                                DecodeCfg<HD>::smem(kDecodeMaxChunkPages));
   });
   if (e != cudaSuccess) return e;
   if (B == 0) return cudaSuccess;
+  const int pg_cap = a.chunk / 64;  // pages one CTA reads
+  if (a.chunk < 64 || a.chunk % 64 || pg_cap > kDecodeMaxChunkPages) return cudaErrorInvalidValue;
   dim3 grid(a.max_splits, a.n_kv, B);
-  e = launch_pdl(attn_decode_kernel<HD>, grid, dim3(128), DecodeCfg<HD>::SMEM, s, tmK, tmV, a);
+  e = launch_pdl(attn_decode_kernel<HD>, grid, dim3(128), DecodeCfg<HD>::smem(pg_cap), s, tmK, tmV, a);
   if (e != cudaSuccess) return e;
   return launch_pdl(attn_combine_kernel<HD>, dim3(B * a.n_q), dim3(HD), 0, s, a);
 }

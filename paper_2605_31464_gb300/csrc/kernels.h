@@ -123,8 +123,7 @@ struct DecodeAttnArgs {
   int n_q, n_kv;
   int64_t layer_row0;
   int64_t layer_vrow0;
-  int chunk;                  // keys per split, multiple of 64; 0: each sequence's pages shared evenly
-                              // among the max_splits CTAs of its row of the grid
+  int chunk;                  // keys per split, multiple of 64 (at most 64 pages)
   int max_splits;
   float* part_o;              // [B][n_kv][max_splits][16][hd] unnormalised partial outputs
   float* part_ml;             // [B][n_kv][max_splits][16][2] (running max in log2 units, sum)

@@ -381,16 +381,6 @@ int decode_chunk(int B, int n_kv, int max_ctx, int sms) {
     if ((int64_t)B * n_kv * ((max_ctx + chunk - 1) / chunk) >= 2 * sms) return chunk;
   return 256;
 }
-// CTAs per (sequence, KV head) in the model's decode step: about GF_DECODE_WAVES times the resident
-// decode-attention CTAs (three per SM) over the B x n_kv pairs, at most `cap` (the partial buffers).
-#ifndef GF_DECODE_WAVES
-#define GF_DECODE_WAVES 2
-#endif
-int decode_splits(int B, int n_kv, int cap, int sms) {
-  const int pairs = B * n_kv;
-  int s = (GF_DECODE_WAVES * 3 * sms + pairs / 2) / pairs;
-  return std::max(1, std::min(s, cap));
-}
 int64_t layer_vrow0(const gf_model* m, int l) { return (int64_t)l * m->num_pages * m->nkv * m->hd; }
 
 
@@ -683,10 +673,8 @@ int decode_impl(gf_model* m, int B, const int32_t* h, const int32_t* ids, float*
     da.n_kv = m->nkv;
     da.layer_row0 = layer_row0(m, l);
     da.layer_vrow0 = layer_vrow0(m, l);
-    // every sequence's context is shared evenly among the same number of CTAs, whatever its length,
-    // sized so that the grid fills the resident CTA slots a whole number of times
-    da.chunk = 0;
-    da.max_splits = decode_splits(B, m->nkv, m->dec_max_splits, m->sms);
+    da.chunk = decode_chunk(B, m->nkv, m->cfg.max_seq, m->sms);
+    da.max_splits = (m->dec_max_splits * m->dec_chunk + da.chunk - 1) / da.chunk;
     da.part_o = m->part_o;
     da.part_ml = m->part_ml;
     da.out = m->dattn;

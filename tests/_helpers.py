@@ -56,28 +56,37 @@ def check_logits(gpu: np.ndarray, ref: np.ndarray, what: str = "logits"):
     return float(err.max())
 
 
-# Full-depth end-to-end logits (28 layers from token ids): the per-element bound above holds for all
-# but a few of the 151,936 logits of a 1.5B-class item.  The bf16 rounding of the activations is what
-# exceeds it: the float64 oracle with bf16 rounding at the GPU path's rounding points (GEMM inputs,
-# rotated q/k, cached v, softmax numerators, attention output, SwiGLU output) misses the bound on 3 of
-# 151,936 prompt logits of 1p5b item 5, by up to 1.10x.  So at full depth at most DEEP_FRAC of the
-# logits may exceed the bound, none by more than DEEP_RATIO, and the mean error must stay within
-# DEEP_MEAN (that emulation: 0.0059).
-DEEP_FRAC = 1e-4
-DEEP_RATIO = 1.5
-DEEP_MEAN = 0.25 * LOGIT_ATOL
+# Full-depth end-to-end logits (28 layers from token ids).  A bf16 data path cannot hold the
+# per-element bound above there: the float64 oracle rounded to bf16 at a bf16 path's rounding points
+# (oracle/bf16_path.py) misses it on 3 of the 151,936 prompt logits of 1p5b item 5 by up to 1.10x, and
+# drifts further at 7B.  So full-depth logits are held to that rounding's own distance from the
+# oracle, from tests/golden/bf16_drift.json (written by tests/golden/make_bf16_drift.py): the
+# root-mean-square error within DRIFT_RMS times it and the largest error within DRIFT_MAX times it.
+DRIFT_RMS = 1.25
+DRIFT_MAX = 1.5
 
 
-def check_logits_deep(gpu: np.ndarray, ref: np.ndarray, what: str = "logits"):
+def bf16_drift(workload: str, item: int) -> dict:
+    import json
+    import os
+    with open(os.path.join(os.path.dirname(__file__), "golden", "bf16_drift.json")) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        if c["workload"] == workload and c["item"] == item:
+            return c
+    raise KeyError(f"no bf16 drift record for {workload} item {item}")
+
+
+def check_logits_deep(gpu: np.ndarray, ref: np.ndarray, drift: dict, what: str = "logits"):
     gpu = np.asarray(gpu, dtype=np.float64)
     err = np.abs(gpu - ref)
-    ratio = err / (LOGIT_ATOL + LOGIT_RTOL * np.abs(ref))
-    n_out = int((ratio > 1).sum())
-    msg = (f"{what}: mean err {err.mean():.4g}, max err {err.max():.4g}, {n_out} of {err.size} beyond the "
-           f"per-element bound, worst {ratio.max():.3f}x")
-    assert err.mean() <= DEEP_MEAN, msg
-    assert n_out <= DEEP_FRAC * err.size, msg
-    assert ratio.max() <= DEEP_RATIO, msg
+    rms = float(np.sqrt(np.mean(err ** 2)))
+    n_out = int((err > LOGIT_ATOL + LOGIT_RTOL * np.abs(ref)).sum())
+    msg = (f"{what}: rms err {rms:.4g} (bf16 rounding alone {drift['rms_err']:.4g}), max err {err.max():.4g} "
+           f"({drift['max_err']:.4g}), {n_out} of {err.size} beyond the per-element bound "
+           f"({drift['outside_elementwise_bound']})")
+    assert rms <= DRIFT_RMS * drift["rms_err"], msg
+    assert err.max() <= DRIFT_MAX * drift["max_err"], msg
     return msg
 
 

@@ -10,10 +10,11 @@ from its token ids:
     of every eighth step (and the last) from a second, eager pass of the same
     batch fed the same tokens.
   The 7B and 14B workloads keep the layer-level checks below.
-  Logits at full depth are held to the stated bound |g - o| <= 3e-2 +
-  2e-2 |o| with the allowance of check_logits_deep (a few logits in 10^5 up to
-  1.5x the bound, mean error under a quarter of 3e-2): an exact bf16 rounding
-  of the same activations misses the per-element bound on a few logits too.
+  Logits at full depth are held to the distance that bf16 rounding alone puts
+  between the float64 oracle and the same forward pass rounded at a bf16
+  path's rounding points (tests/golden/bf16_drift.json; check_logits_deep):
+  that rounding itself misses the per-element bound 3e-2 + 2e-2 |o| on a few
+  logits.  The verdict probabilities keep their 1e-2 bound.
 
 Layer level (test_full_size_workload): the oracle cannot run a whole 7B/14B
 forward pass in seconds, so these tests compare outputs it can compute one by
@@ -38,7 +39,7 @@ import pytest
 
 import oracle
 import synth
-from _helpers import check_logits, check_logits_deep, check_verdict, greedy_agrees, make_model
+from _helpers import bf16_drift, check_logits, check_logits_deep, check_verdict, greedy_agrees, make_model
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -203,11 +204,12 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
                               forced_tokens=toks[item])
     del Wo
     # product path: the logits the verdict reads, the verdict, and every greedy choice
-    print(check_logits_deep(final, ref["step_logits"][n_dec], f"1p5b item {item}: final logits (step {n_dec})"))
+    drift = bf16_drift("1p5b", item)
+    print(check_logits_deep(final, ref["step_logits"][n_dec], drift, f"1p5b item {item}: final logits (step {n_dec})"))
     _check_item_verdict(out, item, ref, w.tau)
     for s in range(n_dec):
         assert greedy_agrees(int(toks[item, s]), ref["step_logits"][s]), f"greedy token of decode input {s}"
     # the eager pass: prompt logits and the logits of the sampled steps
     for s, lg in step_logits.items():
-        print(check_logits_deep(lg, ref["step_logits"][s + 1], f"1p5b item {item}: logits after decode input {s}"))
+        print(check_logits_deep(lg, ref["step_logits"][s + 1], drift, f"1p5b item {item}: logits after decode input {s}"))
 
