@@ -76,9 +76,11 @@ def peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             p = json.load(f)
-        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sus=p["bf16_tflops_sustained"], src="measured")
+        clk = (p.get("clocks_under_load") or {}).get("sm_mhz_median")
+        return dict(hbm=p["hbm_gbs"], bf16=p["bf16_tflops"], bf16_sus=p["bf16_tflops_sustained"], src="measured",
+                    sus_mhz=clk)
     except Exception:
-        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback", sus_mhz=None)
 
 
 def workload_config(w: synth.Workload, world: int) -> dict:
@@ -471,6 +473,12 @@ def run_ours(args):
                  "launches": prof["launches"], "avg_launch_ms": prof["ms"] / max(prof["launches"], 1),
                  "algorithmic_tflop_per_launch": prof["flops"] / max(prof["launches"], 1) / 1e12,
                  "timed_ms": prof["ms"]}
+    if pk.get("sus_mhz") and clk.get("sm_mhz"):
+        # a tensor-bound kernel's rate follows the SM clock: the same ratio at the clock the sustained peak
+        # was measured at (power-capped runs differ in clock)
+        gemm_roof["frac_per_clock"] = gemm_roof["frac"] * pk["sus_mhz"] / clk["sm_mhz"]
+        gemm_roof["clock_note"] = (f"sustained peak measured at a median {pk['sus_mhz']:.0f} MHz SM clock, this run "
+                                   f"at {clk['sm_mhz']:.0f} MHz; frac_per_clock compares them at equal clock")
     dec_gbs = dsteps["bytes"] / (dsteps["ms"] / 1e3) / 1e9 if dsteps["ms"] > 0 else 0.0
     dec_roof = {"bound": "hbm",
                 "kernel": "decode step (CUDA graph of the per-layer kernels), replayed n_decode-1 times per forecast",
