@@ -8,7 +8,9 @@ from its token ids:
     logits the verdict reads, the verdict and defer bit, every one of the 64
     greedy choices against the oracle's logits of that step, and the logits
     of every eighth step (and the last) from a second, eager pass of the same
-    batch fed the same tokens.
+    batch fed the same tokens; and the same item's prompt logits through the
+    shared-incumbent forecast (gf_forecast_batch_shared) and the sampled
+    forecast (gf_forecast_batch_sampled, one repeat) of the whole batch.
   The 7B and 14B workloads keep the layer-level checks below.
   Logits at full depth are held to the distance that bf16 rounding alone puts
   between the float64 oracle and the same forward pass rounded at a bf16
@@ -175,6 +177,20 @@ def _check_item_verdict(out, item, ref, tau):
                   int(out["defer"][item]), ref["p"], ref["conf"], ref["arg"], ref["defer"], tau)
 
 
+def _prompt_logits_other_paths(model, w, item):
+    """Prompt logits of `item` (n_decode = 0) through the shared-incumbent forecast (the incumbent's
+    pages prefilled once) and the sampled forecast (one repeat per item), on the same model."""
+    inc, io, cand, co = synth.prompts(w)
+    cand_d = torch.from_numpy(cand).cuda()
+    sh = model.forecast_batch_shared(torch.from_numpy(inc[:w.inc_len]).cuda(), cand_d, co, 0, w.verdict_ids, w.tau,
+                                     want_tokens=False, want_logits=True)
+    sa = model.forecast_batch_sampled(torch.from_numpy(inc).cuda(), io, cand_d, co, 0, w.verdict_ids, w.tau,
+                                      repeats=1, temperature=1.0, seed=3, want_tokens=False, want_logits=True)
+    torch.cuda.synchronize()
+    model.status()
+    return {"shared-incumbent": sh["logits"][item].cpu().numpy(), "sampled": sa["logits"][item].cpu().numpy()}
+
+
 def test_1p5b_forecast_end_to_end_from_token_ids():
     w = synth.workload("1p5b")
     m, n_dec = w.model, w.n_decode
@@ -195,6 +211,7 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
     torch.cuda.synchronize()
     model.status()
     model.release(handles)
+    others = _prompt_logits_other_paths(model, w, item)
     model.close()
     del model
     torch.cuda.empty_cache()
@@ -212,4 +229,7 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
     # the eager pass: prompt logits and the logits of the sampled steps
     for s, lg in step_logits.items():
         print(check_logits_deep(lg, ref["step_logits"][s + 1], drift, f"1p5b item {item}: logits after decode input {s}"))
+    # the shared-incumbent and sampled forecasts of the same batch: the prompt logits
+    for path, lg in others.items():
+        print(check_logits_deep(lg, ref["step_logits"][0], drift, f"1p5b item {item}: {path} prompt logits"))
 
