@@ -5,6 +5,9 @@ same forward pass rounded to bf16 at a bf16 data path's rounding points (oracle.
 compared: root-mean-square and largest absolute difference of the logits, how many logits fall
 outside |g - o| <= 3e-2 + 2e-2 |o|, and the largest difference of the verdict probabilities.  The
 end-to-end parity tests hold the GPU's own difference from the oracle to a small multiple of these.
+For the cases in SAVE_LOGITS the float64 oracle's prompt logits are also written, as float32, to
+prompt_logits_<workload>_<item>.npy: a whole 7B prompt forward pass takes minutes of host time, so
+the GPU test reads them instead of recomputing them.
 
 Calls only oracle/ and the seeded input generator; runs for tens of minutes on a few host cores
 (two 28-layer prompt forward passes of 4096 and 6144 tokens, twice each).
@@ -29,6 +32,7 @@ import synth  # noqa: E402
 from oracle import bf16_path  # noqa: E402
 
 CASES = [("1p5b", 5), ("7b_prefill", 17)]
+SAVE_LOGITS = {("7b_prefill", 17)}
 OUT = os.path.join(HERE, "bf16_drift.json")
 
 
@@ -47,6 +51,8 @@ def drift(name: str, item: int) -> dict:
         xb = bf16_path.layer_forward_bf16(xb, lw, m, pos)
         print(f"{name} item {item}: layer {l + 1}/{m.layers} ({time.time() - t0:.0f} s)", flush=True)
     ref = oracle.lm_head(x[-1:], W)[0]
+    if (name, item) in SAVE_LOGITS:
+        np.save(os.path.join(HERE, f"prompt_logits_{name}_{item}.npy"), ref.astype(np.float32))
     last = xb[-1:]
     h = bf16_path.bf16_round(last / np.sqrt(np.mean(last * last, axis=-1, keepdims=True) + m.rms_eps) *
                              W.final_norm())

@@ -11,7 +11,11 @@ from its token ids:
     batch fed the same tokens; and the same item's prompt logits through the
     shared-incumbent forecast (gf_forecast_batch_shared) and the sampled
     forecast (gf_forecast_batch_sampled, one repeat) of the whole batch.
-  The 7B and 14B workloads keep the layer-level checks below.
+  - 7b_prefill (32 x 6144, n_decode = 0): item 17's prompt logits and verdict,
+    against oracle logits stored by tests/golden/make_bf16_drift.py (a 7B
+    prompt forward pass takes minutes of host time).
+  The oracle's 256 decode steps of a 7B model, and 7b_decode and 14b_long end
+  to end, are out of its reach in a test; those keep the layer-level checks.
   Logits at full depth are held to the distance that bf16 rounding alone puts
   between the float64 oracle and the same forward pass rounded at a bf16
   path's rounding points (tests/golden/bf16_drift.json; check_logits_deep):
@@ -233,3 +237,26 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
     for path, lg in others.items():
         print(check_logits_deep(lg, ref["step_logits"][0], drift, f"1p5b item {item}: {path} prompt logits"))
 
+
+
+def test_7b_prefill_forecast_end_to_end_from_token_ids():
+    """7b_prefill (32 x 6144) through gf_forecast_batch with n_decode = 0, whole batch: item 17's prompt
+    logits and verdict against the float64 oracle's 28-layer forward pass from the item's token ids.
+    That pass takes minutes of host time, so tests/golden/make_bf16_drift.py (which calls only oracle/)
+    stored its logits in tests/golden/prompt_logits_7b_prefill_17.npy."""
+    import os
+    w = synth.workload("7b_prefill")
+    item = 17
+    ref_logits = np.load(os.path.join(os.path.dirname(__file__), "golden",
+                                      f"prompt_logits_7b_prefill_{item}.npy")).astype(np.float64)
+    assert ref_logits.shape == (w.model.vocab,)
+    model, out = _forecast_whole_batch(w, 0, want_tokens=False)
+    final = out["logits"][item].cpu().numpy()
+    model.close()
+    del model
+    torch.cuda.empty_cache()
+    drift = bf16_drift("7b_prefill", item)
+    print(check_logits_deep(final, ref_logits, drift, f"7b_prefill item {item}: prompt logits"))
+    rp, rc, ra, rd = oracle.verdict(ref_logits[None], w.verdict_ids, w.tau)
+    _check_item_verdict(out, item, {"p": rp[0], "conf": float(rc[0]), "arg": int(ra[0]), "defer": int(rd[0])},
+                        w.tau)
