@@ -199,6 +199,7 @@ __global__ void __launch_bounds__(384, 1) attn_prefill_tc_kernel(const __grid_co
       // -------------------------------------------------------------- MMA issuer
       if (lane == 0) {
         bool ok = mbar_wait(q_full, 0, a.err) && mbar_wait(k0_full, 0, a.err);
+        tc_fence_after();
         bool any = false;
         // operand descriptors of the query tiles and ring slots, built once; an MMA's K step only
         // moves the start address
@@ -242,6 +243,7 @@ __global__ void __launch_bounds__(384, 1) attn_prefill_tc_kernel(const __grid_co
         // one wait per iteration for V(j) and K(j+1), one commit per iteration freeing both slots
         for (int j = 0; j < n_max && ok; ++j) {
           ok = mbar_wait(&vk_full[j & 1], (j >> 1) & 1, a.err);
+          tc_fence_after();
           if (ok && j < n_t[0]) {
             ok = issue_pv(0, j);
             if (ok && j + 1 < n_t[0]) issue_s(0, j + 1);

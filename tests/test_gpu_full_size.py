@@ -11,9 +11,10 @@ from its token ids:
     batch fed the same tokens; and the same item's prompt logits through the
     shared-incumbent forecast (gf_forecast_batch_shared) and the sampled
     forecast (gf_forecast_batch_sampled, one repeat) of the whole batch.
-  - 7b_prefill (32 x 6144, n_decode = 0): item 17's prompt logits and verdict,
-    against oracle logits stored by tests/golden/make_bf16_drift.py (a 7B
-    prompt forward pass takes minutes of host time).
+  - 7b_prefill (32 x 6144) item 17 and 7b_decode (128 ragged prompts) item 11,
+    with n_decode = 0: the prompt logits and verdict, against oracle logits
+    stored by tests/golden/make_bf16_drift.py (a 7B prompt forward pass takes
+    minutes of host time).
   The oracle's 256 decode steps of a 7B model, and 7b_decode and 14b_long end
   to end, are out of its reach in a test; those keep the layer-level checks.
   Logits at full depth are held to the distance that bf16 rounding alone puts
@@ -45,7 +46,8 @@ import pytest
 
 import oracle
 import synth
-from _helpers import bf16_drift, check_logits, check_logits_deep, check_verdict, greedy_agrees, make_model
+from _helpers import (bf16_drift, check_logits, check_logits_deep, check_verdict, greedy_agrees, make_model,
+                      verdict_tol_deep)
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -176,9 +178,9 @@ def _forecast_whole_batch(w, n_decode, want_tokens):
     return model, out
 
 
-def _check_item_verdict(out, item, ref, tau):
+def _check_item_verdict(out, item, ref, tau, p_atol):
     check_verdict(out["p"][item].cpu().numpy(), float(out["conf"][item]), int(out["arg"][item]),
-                  int(out["defer"][item]), ref["p"], ref["conf"], ref["arg"], ref["defer"], tau)
+                  int(out["defer"][item]), ref["p"], ref["conf"], ref["arg"], ref["defer"], tau, p_atol=p_atol)
 
 
 def _prompt_logits_other_paths(model, w, item):
@@ -227,7 +229,7 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
     # product path: the logits the verdict reads, the verdict, and every greedy choice
     drift = bf16_drift("1p5b", item)
     print(check_logits_deep(final, ref["step_logits"][n_dec], drift, f"1p5b item {item}: final logits (step {n_dec})"))
-    _check_item_verdict(out, item, ref, w.tau)
+    _check_item_verdict(out, item, ref, w.tau, verdict_tol_deep(drift, ref["p"]))
     for s in range(n_dec):
         assert greedy_agrees(int(toks[item, s]), ref["step_logits"][s]), f"greedy token of decode input {s}"
     # the eager pass: prompt logits and the logits of the sampled steps
@@ -239,24 +241,27 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
 
 
 
-def test_7b_prefill_forecast_end_to_end_from_token_ids():
-    """7b_prefill (32 x 6144) through gf_forecast_batch with n_decode = 0, whole batch: item 17's prompt
-    logits and verdict against the float64 oracle's 28-layer forward pass from the item's token ids.
-    That pass takes minutes of host time, so tests/golden/make_bf16_drift.py (which calls only oracle/)
-    stored its logits in tests/golden/prompt_logits_7b_prefill_17.npy."""
+@pytest.mark.parametrize("name,item", [("7b_prefill", 17), ("7b_decode", 11)])
+def test_7b_forecast_prompt_logits_end_to_end_from_token_ids(name, item):
+    """7b_prefill (32 x 6144) and 7b_decode (128 ragged prompts of U[1024, 2048] ids) through
+    gf_forecast_batch with n_decode = 0, whole batch: one item's prompt logits and verdict against the
+    float64 oracle's 28-layer pass from the item's token ids.  That pass takes minutes of host time, so
+    tests/golden/make_bf16_drift.py (which calls only oracle/) stored its logits in
+    tests/golden/prompt_logits_<workload>_<item>.npy."""
     import os
-    w = synth.workload("7b_prefill")
-    item = 17
+    w = synth.workload(name)
     ref_logits = np.load(os.path.join(os.path.dirname(__file__), "golden",
-                                      f"prompt_logits_7b_prefill_{item}.npy")).astype(np.float64)
+                                      f"prompt_logits_{name}_{item}.npy")).astype(np.float64)
     assert ref_logits.shape == (w.model.vocab,)
     model, out = _forecast_whole_batch(w, 0, want_tokens=False)
     final = out["logits"][item].cpu().numpy()
     model.close()
     del model
     torch.cuda.empty_cache()
-    drift = bf16_drift("7b_prefill", item)
-    print(check_logits_deep(final, ref_logits, drift, f"7b_prefill item {item}: prompt logits"))
+    drift = bf16_drift(name, item)
+    print(check_logits_deep(final, ref_logits, drift, f"{name} item {item}: prompt logits"))
     rp, rc, ra, rd = oracle.verdict(ref_logits[None], w.verdict_ids, w.tau)
+    tol = verdict_tol_deep(drift, rp[0])
+    print(f"{name} item {item}: verdict p {out['p'][item].cpu().numpy()} vs oracle {rp[0]} (tolerance {tol:.4f})")
     _check_item_verdict(out, item, {"p": rp[0], "conf": float(rc[0]), "arg": int(ra[0]), "defer": int(rd[0])},
-                        w.tau)
+                        w.tau, tol)
