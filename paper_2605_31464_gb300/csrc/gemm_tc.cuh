@@ -91,10 +91,12 @@ struct GemmCfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-  static constexpr int STAGES_FIT = (220 * 1024) / STAGE_BYTES;
+  // non-swapped tiles keep 18 KB for the epilogue's staging tiles (4 warps x [32 rows][36 floats])
+  static constexpr int EPI_BYTES = SWAP ? 0 : 4 * 32 * 36 * 4;
+  static constexpr int STAGES_FIT = ((SWAP ? 220 : 200) * 1024) / STAGE_BYTES;
   static constexpr int STAGES = STAGES_FIT > 12 ? 12 : STAGES_FIT;
   static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // two accumulator buffers
-  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/;
+  static constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 /*align*/ + 256 /*barriers*/ + EPI_BYTES;
   static constexpr int THREADS = 192;
 };
 
@@ -178,6 +180,7 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* acc_empty = acc_full + 2;
   uint64_t* mma_done = acc_empty + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(mma_done + 1);
+  float* epi_smem = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [4][32][36] (non-swapped)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -498,60 +501,69 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       } else if (MODE == kAddF32) {
-        // the residual chunk of the next 32 columns is loaded while this chunk is added and stored
-        float ss = 0.f;
-        float* res_row = reinterpret_cast<float*>(p.out) + (int64_t)row * p.ldo + n_blk * BN;
+        // TMEM hands each thread one row (lane = row), so a warp's global accesses would each touch 32
+        // rows.  Each warp stages its 32 rows x 32 columns through shared memory instead and lane l then
+        // handles columns 4 (l % 8) .. + 3 of rows 4 k + l / 8 (k = 0..7): an access covers four whole
+        // 128-byte row pieces.  Row sums of squares are reduced over the eight lanes of a row.
+        float* stile = epi_smem + quarter * (32 * 36);
+        const int sub = lane & 7, rq = lane >> 3;
+        const int row0 = m_blk * C::BM + quarter * 32;
         const int ncols = min(BN, p.N - n_blk * BN);
-        float4 cur[8], nxt[8];
-        if (row_ok && ncols > 0) {
+        float* res_base = reinterpret_cast<float*>(p.out);
+        float ss[8];
 #pragma unroll
-          for (int i = 0; i < 8; ++i) cur[i] = reinterpret_cast<const float4*>(res_row)[i];
-        }
+        for (int k = 0; k < 8; ++k) ss[k] = 0.f;
 #pragma unroll 1
-        for (int c = 0; c < BN; c += 32) {
+        for (int c = 0; c < ncols; c += 32) {
           uint32_t r[32];
           tmem_ld32(taddr + c, r);
-          const bool have_next = row_ok && c + 32 < ncols;
-          if (have_next) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) nxt[i] = reinterpret_cast<const float4*>(res_row + c + 32)[i];
-          }
           tmem_ld_wait();
-          const int col = n_blk * BN + c;
-          if (row_ok && c < ncols) {
-            float4* dst = reinterpret_cast<float4*>(res_row + c);
-            float x[32];
+          float4* srow = reinterpret_cast<float4*>(stile + lane * 36);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              x[4 * i] = cur[i].x + __uint_as_float(r[4 * i]);
-              x[4 * i + 1] = cur[i].y + __uint_as_float(r[4 * i + 1]);
-              x[4 * i + 2] = cur[i].z + __uint_as_float(r[4 * i + 2]);
-              x[4 * i + 3] = cur[i].w + __uint_as_float(r[4 * i + 3]);
-            }
+          for (int i = 0; i < 8; ++i)
+            srow[i] = make_float4(__uint_as_float(r[4 * i]), __uint_as_float(r[4 * i + 1]), __uint_as_float(r[4 * i + 2]),
+                                  __uint_as_float(r[4 * i + 3]));
+          __syncwarp();
+          const int col = n_blk * BN + c + 4 * sub;
+          float4 x[8];
 #pragma unroll
-            for (int i = 0; i < 8; ++i) dst[i] = make_float4(x[4 * i], x[4 * i + 1], x[4 * i + 2], x[4 * i + 3]);
-            if (p.norm_out) {
-              const float4* g4 = reinterpret_cast<const float4*>(p.norm_gain + col);
-              uint32_t pk[16];
+          for (int k = 0; k < 8; ++k) {
+            const int row = row0 + 4 * k + rq;
+            x[k] = row < p.M ? *reinterpret_cast<const float4*>(res_base + (int64_t)row * p.ldo + col)
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+          }
+          float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+          if (p.norm_out) g = *reinterpret_cast<const float4*>(p.norm_gain + col);
 #pragma unroll
-              for (int i = 0; i < 8; ++i) {
-                const float4 g = g4[i];
-                ss += x[4 * i] * x[4 * i] + x[4 * i + 1] * x[4 * i + 1] + x[4 * i + 2] * x[4 * i + 2] +
-                      x[4 * i + 3] * x[4 * i + 3];
-                pk[2 * i] = pack_bf16(x[4 * i] * g.x, x[4 * i + 1] * g.y);
-                pk[2 * i + 1] = pack_bf16(x[4 * i + 2] * g.z, x[4 * i + 3] * g.w);
+          for (int k = 0; k < 8; ++k) {
+            const int row = row0 + 4 * k + rq;
+            const float4 a = reinterpret_cast<const float4*>(stile + (4 * k + rq) * 36)[sub];
+            x[k].x += a.x;
+            x[k].y += a.y;
+            x[k].z += a.z;
+            x[k].w += a.w;
+            if (row < p.M) {
+              *reinterpret_cast<float4*>(res_base + (int64_t)row * p.ldo + col) = x[k];
+              if (p.norm_out) {
+                ss[k] += x[k].x * x[k].x + x[k].y * x[k].y + x[k].z * x[k].z + x[k].w * x[k].w;
+                *reinterpret_cast<uint2*>(p.norm_out + (int64_t)row * p.ld_norm + col) =
+                    make_uint2(pack_bf16(x[k].x * g.x, x[k].y * g.y), pack_bf16(x[k].z * g.z, x[k].w * g.w));
               }
-              uint4* nd = reinterpret_cast<uint4*>(p.norm_out + (int64_t)row * p.ld_norm + col);
-#pragma unroll
-              for (int q = 0; q < 4; ++q) nd[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
             }
           }
-          if (have_next) {
+          __syncwarp();  // the next chunk overwrites the staging tile
+        }
+        if (p.norm_out) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) cur[i] = nxt[i];
+          for (int k = 0; k < 8; ++k) {
+            float v = ss[k];
+            v += __shfl_xor_sync(0xffffffffu, v, 1);
+            v += __shfl_xor_sync(0xffffffffu, v, 2);
+            v += __shfl_xor_sync(0xffffffffu, v, 4);
+            const int row = row0 + 4 * k + rq;
+            if (sub == 0 && row < p.M) atomicAdd(p.norm_ss + row, v);
           }
         }
-        if (p.norm_out && row_ok) atomicAdd(p.norm_ss + row, ss);
       } else {
 #pragma unroll 1
         for (int c = 0; c < BN; c += 32) {
