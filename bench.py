@@ -36,7 +36,7 @@ import synth  # noqa: E402
 # 113 prefill GEMM launches of one forecast (28 layers x 4 + the LM head),
 # captured on 4 x 6144 tokens with two layers and scaled by the 8x rows (the
 # traffic of these GEMMs grows in proportion to the rows).
-NCU_TRAFFIC = {"7b_prefill": 18.41e9}
+NCU_TRAFFIC = {"7b_prefill": 18.49e9}
 
 
 def parse_args():
