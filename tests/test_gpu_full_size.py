@@ -265,3 +265,37 @@ def test_7b_forecast_prompt_logits_end_to_end_from_token_ids(name, item):
     print(f"{name} item {item}: verdict p {out['p'][item].cpu().numpy()} vs oracle {rp[0]} (tolerance {tol:.4f})")
     _check_item_verdict(out, item, {"p": rp[0], "conf": float(rc[0]), "arg": int(ra[0]), "defer": int(rd[0])},
                         w.tau, tol)
+
+
+def test_7b_prefill_decode_steps_fed_the_oracle_tokens():
+    """7b_prefill: the whole 32 x 6144 batch prefilled and then decoded for 8 steps in the benchmark's
+    launch configuration, every sequence fed the float64 oracle's own greedy tokens for item 17; item 17's
+    logits after decode inputs 3 and 7 against the oracle's (tests/golden/decode_steps_7b_prefill_17.npz,
+    written by tests/golden/make_decode_steps.py, which calls only oracle/)."""
+    import os
+    w = synth.workload("7b_prefill")
+    m, item = w.model, 17
+    g = np.load(os.path.join(os.path.dirname(__file__), "golden", f"decode_steps_7b_prefill_{item}.npz"))
+    toks = g["tokens"]
+    ids, off = synth.packed_prompts(w)
+    lens = np.diff(off)
+    model = make_model(m, max_batch=w.batch, max_seq=int(lens.max()) + len(toks) + 1,
+                       max_prefill_tokens=int(off[-1]))
+    handles, _, _ = model.prefill(torch.from_numpy(ids).cuda(), off)
+    got = {}
+    for s in range(len(toks)):
+        step_ids = torch.full((w.batch,), int(toks[s]), dtype=torch.int32, device="cuda")
+        lg, _ = model.decode_step(handles, step_ids, want_logits=f"logits_{s + 1}" in g.files)
+        if f"logits_{s + 1}" in g.files:
+            got[s + 1] = lg[item].cpu().numpy()
+    torch.cuda.synchronize()
+    model.status()
+    model.release(handles)
+    model.close()
+    del model
+    torch.cuda.empty_cache()
+    assert sorted(got) == [4, 8]
+    drift = bf16_drift("7b_prefill", item)
+    for s, lg in got.items():
+        print(check_logits_deep(lg, g[f"logits_{s}"].astype(np.float64), drift,
+                                f"7b_prefill item {item}: logits after decode input {s - 1}"))
