@@ -267,15 +267,17 @@ def test_7b_forecast_prompt_logits_end_to_end_from_token_ids(name, item):
                         w.tau, tol)
 
 
-def test_7b_prefill_decode_steps_fed_the_oracle_tokens():
-    """7b_prefill: the whole 32 x 6144 batch prefilled and then decoded for 8 steps in the benchmark's
-    launch configuration, every sequence fed the float64 oracle's own greedy tokens for item 17; item 17's
-    logits after decode inputs 3 and 7 against the oracle's (tests/golden/decode_steps_7b_prefill_17.npz,
-    written by tests/golden/make_decode_steps.py, which calls only oracle/)."""
+@pytest.mark.parametrize("name,item", [("7b_prefill", 17), ("7b_decode", 11)])
+def test_7b_decode_steps_fed_the_oracle_tokens(name, item):
+    """7b_prefill (32 x 6144) and 7b_decode (128 ragged prompts): the whole batch prefilled and then decoded
+    for 8 steps in the benchmark's launch configuration, every sequence fed the float64 oracle's own greedy
+    tokens for one item; that item's logits after decode inputs 3 and 7 against the oracle's
+    (tests/golden/decode_steps_<workload>_<item>.npz, written by tests/golden/make_decode_steps.py, which
+    calls only oracle/)."""
     import os
-    w = synth.workload("7b_prefill")
-    m, item = w.model, 17
-    g = np.load(os.path.join(os.path.dirname(__file__), "golden", f"decode_steps_7b_prefill_{item}.npz"))
+    w = synth.workload(name)
+    m = w.model
+    g = np.load(os.path.join(os.path.dirname(__file__), "golden", f"decode_steps_{name}_{item}.npz"))
     toks = g["tokens"]
     ids, off = synth.packed_prompts(w)
     lens = np.diff(off)
@@ -295,7 +297,7 @@ def test_7b_prefill_decode_steps_fed_the_oracle_tokens():
     del model
     torch.cuda.empty_cache()
     assert sorted(got) == [4, 8]
-    drift = bf16_drift("7b_prefill", item)
+    drift = bf16_drift(name, item)
     for s, lg in got.items():
         print(check_logits_deep(lg, g[f"logits_{s}"].astype(np.float64), drift,
-                                f"7b_prefill item {item}: logits after decode input {s - 1}"))
+                                f"{name} item {item}: logits after decode input {s - 1}"))
