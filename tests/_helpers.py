@@ -115,8 +115,9 @@ def check_verdict(gpu_p, gpu_conf, gpu_arg, gpu_defer, ref_p, ref_conf, ref_arg,
 # Full-depth verdicts.  p_i = softmax over the verdict ids of the final logits, so a logit error e moves
 # p_i by about p_i (1 - p_i) (e_i - e_j) (two ids); with the rms logit error the drift reading allows
 # (DRIFT_RMS times that of bf16 rounding alone) the difference of two logits' errors has an rms of about
-# sqrt(2) times it.  The verdict is held to twice that standard deviation, and never looser than 1e-2
-# needs: at 1.5B depth this is the 1e-2 bound itself, at 7B depth about 2e-2.
+# sqrt(2) times it.  The verdict is held to three times that standard deviation, and never looser than
+# 1e-2 needs: at 1.5B depth this is the 1e-2 bound itself, at 7B depth about 3e-2 (the logits' own
+# bound allows up to about 9e-2: 1/4 of twice the largest logit error).
 def verdict_tol_deep(drift: dict, ref_p) -> float:
     sens = float(np.max(np.asarray(ref_p) * (1.0 - np.asarray(ref_p))))
-    return max(P_ATOL, 2.0 * sens * np.sqrt(2.0) * DRIFT_RMS * drift["rms_err"])
+    return max(P_ATOL, 3.0 * sens * np.sqrt(2.0) * DRIFT_RMS * drift["rms_err"])

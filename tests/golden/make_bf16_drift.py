@@ -9,8 +9,8 @@ For the cases in SAVE_LOGITS the float64 oracle's prompt logits are also written
 prompt_logits_<workload>_<item>.npy: a whole 7B prompt forward pass takes minutes of host time, so
 the GPU test reads them instead of recomputing them.
 
-Calls only oracle/ and the seeded input generator; runs for about an hour on a few host cores
-(28-layer prompt forward passes of 4096, 6144 and 2038 tokens, twice each).
+Calls only oracle/ and the seeded input generator; runs for about two hours on eight host cores
+(28-layer prompt forward passes of 4096, 2 x 6144, 2038 and 1029 tokens, twice each).
 
     python tests/golden/make_bf16_drift.py [workload:item ...]
 """
@@ -31,8 +31,8 @@ import oracle  # noqa: E402
 import synth  # noqa: E402
 from oracle import bf16_path  # noqa: E402
 
-CASES = [("1p5b", 5), ("7b_prefill", 17), ("7b_decode", 11)]
-SAVE_LOGITS = {("7b_prefill", 17), ("7b_decode", 11)}
+CASES = [("1p5b", 5), ("7b_prefill", 17), ("7b_prefill", 3), ("7b_decode", 11), ("7b_decode", 76)]
+SAVE_LOGITS = {("7b_prefill", 17), ("7b_prefill", 3), ("7b_decode", 11), ("7b_decode", 76)}
 OUT = os.path.join(HERE, "bf16_drift.json")
 
 

@@ -11,17 +11,19 @@ from its token ids:
     batch fed the same tokens; and the same item's prompt logits through the
     shared-incumbent forecast (gf_forecast_batch_shared) and the sampled
     forecast (gf_forecast_batch_sampled, one repeat) of the whole batch.
-  - 7b_prefill (32 x 6144) item 17 and 7b_decode (128 ragged prompts) item 11,
-    with n_decode = 0: the prompt logits and verdict, against oracle logits
-    stored by tests/golden/make_bf16_drift.py (a 7B prompt forward pass takes
-    minutes of host time).
-  The oracle's 256 decode steps of a 7B model, and 7b_decode and 14b_long end
-  to end, are out of its reach in a test; those keep the layer-level checks.
+  - 7b_prefill (32 x 6144) items 17 and 3 and 7b_decode (128 ragged prompts)
+    items 11 and 76, with n_decode = 0: the prompt logits and verdicts, against
+    oracle logits stored by tests/golden/make_bf16_drift.py (a 7B prompt
+    forward pass takes minutes of host time); and 8 decode steps of items 17
+    and 11 fed the oracle's own greedy tokens.
+  All 256 (2048) decode steps of a 7B model, and 14b_long end to end, are out
+  of the oracle's reach; those keep the layer-level checks below.
   Logits at full depth are held to the distance that bf16 rounding alone puts
   between the float64 oracle and the same forward pass rounded at a bf16
   path's rounding points (tests/golden/bf16_drift.json; check_logits_deep):
   that rounding itself misses the per-element bound 3e-2 + 2e-2 |o| on a few
-  logits.  The verdict probabilities keep their 1e-2 bound.
+  logits.  The verdict probabilities follow from those logits: they are held
+  to max(1e-2, three times the spread that logit drift implies) (verdict_tol_deep).
 
 Layer level (test_full_size_workload): the oracle cannot run a whole 7B/14B
 forward pass in seconds, so these tests compare outputs it can compute one by
@@ -241,30 +243,31 @@ def test_1p5b_forecast_end_to_end_from_token_ids():
 
 
 
-@pytest.mark.parametrize("name,item", [("7b_prefill", 17), ("7b_decode", 11)])
-def test_7b_forecast_prompt_logits_end_to_end_from_token_ids(name, item):
-    """7b_prefill (32 x 6144) and 7b_decode (128 ragged prompts of U[1024, 2048] ids) through
-    gf_forecast_batch with n_decode = 0, whole batch: one item's prompt logits and verdict against the
-    float64 oracle's 28-layer pass from the item's token ids.  That pass takes minutes of host time, so
-    tests/golden/make_bf16_drift.py (which calls only oracle/) stored its logits in
-    tests/golden/prompt_logits_<workload>_<item>.npy."""
+@pytest.mark.parametrize("name,items", [("7b_prefill", (17, 3)), ("7b_decode", (11, 76))])
+def test_7b_forecast_prompt_logits_end_to_end_from_token_ids(name, items):
+    """7b_prefill (32 x 6144) and 7b_decode (128 ragged prompts of U[1024, 2048] ids; item 76 is the
+    shortest, 1029 tokens) through gf_forecast_batch with n_decode = 0, whole batch: two items' prompt
+    logits and verdicts against the float64 oracle's 28-layer pass from each item's token ids.  That pass
+    takes minutes of host time, so tests/golden/make_bf16_drift.py (which calls only oracle/) stored its
+    logits in tests/golden/prompt_logits_<workload>_<item>.npy."""
     import os
     w = synth.workload(name)
-    ref_logits = np.load(os.path.join(os.path.dirname(__file__), "golden",
-                                      f"prompt_logits_{name}_{item}.npy")).astype(np.float64)
-    assert ref_logits.shape == (w.model.vocab,)
     model, out = _forecast_whole_batch(w, 0, want_tokens=False)
-    final = out["logits"][item].cpu().numpy()
+    finals = {item: out["logits"][item].cpu().numpy() for item in items}
     model.close()
     del model
     torch.cuda.empty_cache()
-    drift = bf16_drift(name, item)
-    print(check_logits_deep(final, ref_logits, drift, f"{name} item {item}: prompt logits"))
-    rp, rc, ra, rd = oracle.verdict(ref_logits[None], w.verdict_ids, w.tau)
-    tol = verdict_tol_deep(drift, rp[0])
-    print(f"{name} item {item}: verdict p {out['p'][item].cpu().numpy()} vs oracle {rp[0]} (tolerance {tol:.4f})")
-    _check_item_verdict(out, item, {"p": rp[0], "conf": float(rc[0]), "arg": int(ra[0]), "defer": int(rd[0])},
-                        w.tau, tol)
+    for item in items:
+        ref_logits = np.load(os.path.join(os.path.dirname(__file__), "golden",
+                                          f"prompt_logits_{name}_{item}.npy")).astype(np.float64)
+        assert ref_logits.shape == (w.model.vocab,)
+        drift = bf16_drift(name, item)
+        print(check_logits_deep(finals[item], ref_logits, drift, f"{name} item {item}: prompt logits"))
+        rp, rc, ra, rd = oracle.verdict(ref_logits[None], w.verdict_ids, w.tau)
+        tol = verdict_tol_deep(drift, rp[0])
+        print(f"{name} item {item}: verdict p {out['p'][item].cpu().numpy()} vs oracle {rp[0]} (tolerance {tol:.4f})")
+        _check_item_verdict(out, item, {"p": rp[0], "conf": float(rc[0]), "arg": int(ra[0]), "defer": int(rd[0])},
+                            w.tau, tol)
 
 
 @pytest.mark.parametrize("name,item", [("7b_prefill", 17), ("7b_decode", 11)])
