@@ -31,7 +31,7 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 # DRAM bytes per launch of the dominant kernel, from an ncu capture of the
-# same kernel build, or None when no capture of this build exists.
+# current kernels (the same source), or None when no such capture exists.
 # 7b_prefill: dram__bytes_read + dram__bytes_write per launch, averaged over the
 # 113 prefill GEMM launches of one forecast (28 layers x 4 + the LM head),
 # captured on 4 x 6144 tokens with two layers and scaled by the 8x rows (the
